@@ -1,0 +1,162 @@
+"""Pins for oracle.calibrate / compress / attention against what the paper and the
+mathematics fix: Eckart-Young truncation loss (Lemma trunc), exact reconstruction at r = d,
+the orthogonal error split of Lemma head-dist (step 1), the KL weight ordering (Sec. 4), the
+rank-space decode identity, and the special cases T = 1, r_K = 0, r_V = 0 and near-lossless
+codes."""
+import math
+
+import numpy as np
+import pytest
+import scipy.special
+
+from oracle import attention, calibrate, compress, hadamard, quantizer
+from paper_2609_24298_gb300 import synth
+
+
+def head(seed=0, alpha=(0.5, 2.0), n=512):
+    src = synth.HeadSource(99, 0, seed, 0, alpha)
+    return src, src.calibration(n)
+
+
+def test_covariance_and_eigenbasis():
+    _, x = head(1)
+    cal = calibrate.calibrate_head(x)
+    lam, U = cal["lam"], cal["U"]
+    assert np.all(np.diff(lam) <= 0)
+    assert np.abs(U.T @ U - np.eye(128)).max() < 1e-12
+    assert np.abs(U @ np.diag(lam) @ U.T - cal["cov"]).max() < 1e-10 * lam[0]
+    assert np.abs(cal["cov"] - np.cov(np.asarray(x, np.float64).T, bias=True)).max() < 1e-10 * lam[0]
+    for j in range(128):
+        k = np.argmax(np.abs(U[:, j]))
+        assert U[k, j] > 0
+
+
+@pytest.mark.parametrize("r", [0, 2, 16, 50, 128])
+def test_eckart_young_on_calibration_set(r):
+    _, x = head(2)
+    cal = calibrate.calibrate_head(x)
+    xc = np.asarray(x, float) - cal["mu"]
+    Ur = cal["U"][:, :r]
+    resid = xc - xc @ Ur @ Ur.T
+    assert abs(np.mean(np.sum(resid ** 2, 1)) - cal["lam"][r:].sum()) < 1e-9 * cal["lam"].sum()
+
+
+def test_full_rank_projection_reconstructs():
+    _, x = head(3)
+    cal = calibrate.calibrate_head(x)
+    s = synth.hadamard_signs(99, 0, 3, 0)
+    W = calibrate.fuse_basis(cal["U"], 128, s)
+    y = compress.project(x, W, cal["mu"])
+    assert np.abs(y @ W.T + cal["mu"] - x).max() < 1e-12 * np.abs(x).max()
+
+
+def test_orthogonal_error_split():
+    """||x - x^||^2 = ||xi_1||^2 + ||xi_2||^2 per sample (Lemma head-dist, step 1)."""
+    _, x = head(4)
+    cal = calibrate.calibrate_head(x)
+    r, b = 40, 3
+    s = synth.hadamard_signs(99, 0, 4, 0)
+    p = calibrate.head_params(cal, r, b, s)
+    W = p["W"].astype(np.float64)
+    u, codes = compress.compress(x, p["W"], p["mu"], p["delta"], b)
+    xh = attention.reconstruct(codes, p["W"], p["delta"], b, p["mu"])
+    xc = np.asarray(x, float) - p["mu"].astype(float)
+    xi1 = xc - xc @ W @ W.T
+    y = xc @ W
+    xi2 = (y - quantizer.dequantize(codes, float(p["delta"]), b)) @ W.T
+    lhs = np.sum((x - xh) ** 2, 1)
+    rhs = np.sum(xi1 ** 2, 1) + np.sum(xi2 ** 2, 1)
+    # W is fp32-rounded, so orthogonality holds to ~1e-7
+    assert np.abs(lhs - rhs).max() < 1e-5 * lhs.max()
+
+
+def test_kl_weights_and_reorder():
+    _, x = head(5)
+    qc = synth.calibration_queries(99, 0, 5, 4, 256, (0.5, 2.0))
+    cal = calibrate.calibrate_head(x, qc)
+    assert np.all(np.diff(cal["w"]) <= 0)
+    # w_i = E[(u_i . q)^2] * lambda_i for each reordered column
+    qs = qc.reshape(-1, 128).astype(float)
+    for j in (0, 7, 127):
+        sq = np.mean((qs @ cal["U"][:, j]) ** 2)
+        lam_j = cal["U"][:, j] @ cal["cov"] @ cal["U"][:, j]
+        assert abs(cal["w"][j] - sq * lam_j) < 1e-9 * cal["w"][0]
+        assert abs(cal["lam"][j] - lam_j) < 1e-9 * cal["lam"].max()
+
+
+def test_hadamard_equalises_rotated_variance():
+    """After fusion, every retained channel of a power-of-two block has the mean retained
+    eigenvalue as variance on the calibration set (App. A.1)."""
+    _, x = head(6)
+    cal = calibrate.calibrate_head(x)
+    s = synth.hadamard_signs(99, 0, 6, 0)
+    W = calibrate.fuse_basis(cal["U"], 64, s)
+    y = compress.project(x, W, cal["mu"])
+    assert np.allclose(y.var(0), cal["lam"][:64].mean(), rtol=1e-9)
+
+
+def make_params(src, r, b):
+    cal = calibrate.calibrate_head(src.calibration(512))
+    s = synth.hadamard_signs(*src.key)
+    return calibrate.head_params(cal, r, b, s)
+
+
+def setup_decode(T, rk, bk, rv, bv, G=4, seed=10):
+    srck = synth.HeadSource(99, 1, seed, 0, (0.5, 2.0))
+    srcv = synth.HeadSource(99, 1, seed, 1, (0.5, 2.0))
+    pk = make_params(srck, rk, bk)
+    pv = make_params(srcv, rv, bv)
+    xk, xv = srck.tokens(T), srcv.tokens(T)
+    _, ck = compress.compress(xk, pk["W"], pk["mu"], pk["delta"], bk)
+    _, cv = compress.compress(xv, pv["W"], pv["mu"], pv["delta"], bv)
+    q = synth.decode_queries(99, 0, seed, 1, G)[0]
+    return q, ck, cv, pk, pv, xk, xv
+
+
+@pytest.mark.parametrize("rk,bk,rv,bv", [(32, 3, 64, 2), (128, 1, 16, 8), (2, 5, 2, 1), (100, 2, 128, 4)])
+def test_rank_space_equals_plain_definition(rk, bk, rv, bv):
+    q, ck, cv, pk, pv, _, _ = setup_decode(300, rk, bk, rv, bv)
+    a = attention.decode(q, ck, cv, pk, pv)
+    b = attention.rank_space(q, ck, cv, pk, pv)
+    assert np.abs(a - b).max() < 1e-12 * np.abs(a).max()
+
+
+def test_softmax_matches_library():
+    g = np.random.default_rng(0)
+    q, K, V = g.standard_normal((4, 128)), g.standard_normal((50, 128)), g.standard_normal((50, 128))
+    p = scipy.special.softmax(q @ K.T / math.sqrt(128), axis=1)
+    assert np.abs(attention.softmax_attend(q, K, V) - p @ V).max() < 1e-13
+
+
+def test_single_token_returns_its_value():
+    q, ck, cv, pk, pv, _, _ = setup_decode(1, 32, 3, 32, 3)
+    o = attention.decode(q, ck, cv, pk, pv)
+    v0 = attention.reconstruct(cv, pv["W"], pv["delta"], 3, pv["mu"])[0]
+    assert np.abs(o - v0[None, :]).max() < 1e-12
+
+
+def test_rank_zero_key_gives_uniform_attention():
+    q, ck, cv, pk, pv, _, _ = setup_decode(77, 0, 0, 32, 3)
+    o = attention.decode(q, ck, cv, pk, pv)
+    V = attention.reconstruct(cv, pv["W"], pv["delta"], 3, pv["mu"])
+    assert np.abs(o - V.mean(0)[None, :]).max() < 1e-12
+    assert np.abs(attention.rank_space(q, ck, cv, pk, pv) - o).max() < 1e-12
+
+
+def test_rank_zero_value_gives_mean():
+    q, ck, cv, pk, pv, _, _ = setup_decode(77, 32, 3, 0, 0)
+    o = attention.rank_space(q, ck, cv, pk, pv)
+    assert np.abs(o - pv["mu"][None, :].astype(float)).max() == 0
+
+
+def test_near_lossless_codes_approach_exact_attention():
+    T = 400
+    q, ck, cv, pk, pv, xk, xv = setup_decode(T, 128, 8, 128, 8)
+    o = attention.decode(q, ck, cv, pk, pv)
+    exact = attention.softmax_attend(q, xk, xv)
+    rel = np.abs(o - exact).max() / np.abs(exact).max()
+    assert rel < 0.05
+    # and with coarse codes the error grows
+    q, ck, cv, pk, pv, xk, xv = setup_decode(T, 128, 2, 128, 2)
+    rel2 = np.abs(attention.decode(q, ck, cv, pk, pv) - exact).max() / np.abs(exact).max()
+    assert rel2 > rel
