@@ -7,7 +7,7 @@ with it.
 
 Every function restates, in plain slow numpy, a step the paper defines; each cites the
 section / equation / table it follows.  Where the paper is silent or ambiguous the
-reading taken is stated in the docstring (the same readings are listed in the design doc).
+reading taken is stated in the docstring.
 
 Modules
   hadamard   fused Walsh-Hadamard rotation with the random sign flip (Sec. 3.4)

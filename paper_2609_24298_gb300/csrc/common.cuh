@@ -1,0 +1,208 @@
+// Device helpers for libcobra's kernels (sm_103a): PTX wrappers and the register-level
+// unpacking of packed code pieces into f16 MMA operands.
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+namespace cobra {
+
+// ---------------------------------------------------------------------------------------
+// status word: bit 0 = a bounded wait expired
+// ---------------------------------------------------------------------------------------
+__device__ unsigned int g_status;
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// ---------------------------------------------------------------------------------------
+// mbarrier + bulk async copy (global -> shared, completion counted in bytes)
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_inval(uint32_t bar) {
+  asm volatile("mbarrier.inval.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Wait for phase `parity` of `bar` to complete, giving up after ~`limit_ns` nanoseconds.
+__device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255) == 255 && globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------------------
+// legacy warp-level MMA (operands in registers) and 8x8 transposition
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ void mma_f16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                        uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
+  uint32_t y;
+  asm("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+  return y;
+}
+__device__ __forceinline__ uint32_t pack_f16(float lo_col, float hi_col) {
+  __half2 h = __floats2half2_rn(lo_col, hi_col);  // .x -> low 16 bits
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// ---------------------------------------------------------------------------------------
+// Unpacking one piece (b little-endian words, 32 codes) into 16 f16x2 registers.
+//
+// Register rho holds code (rho, 0) in its low half and code (rho, 1) in its high half, as
+// the f16 value off(rho) + code: the code is masked into mantissa bits [k, k+b) of a half
+// whose exponent field makes the value 2^(10-k) + code (k + b <= 10), so one AND/OR (plus
+// at most a shift) yields two codes.  off(rho) = 2^(10-k) is removed after the MMA.
+// ---------------------------------------------------------------------------------------
+__host__ __device__ constexpr uint32_t magic2(int k) {
+  return ((uint32_t)(25 - k) << 10) | ((uint32_t)(25 - k) << 26);
+}
+__host__ __device__ constexpr uint32_t pair_mask(int nbits, int k) {
+  return (((1u << nbits) - 1u) << k) * 0x00010001u;
+}
+
+template <int B>
+struct Window {
+  // mantissa position used for register rho, and the matching offset 2^(10-k)
+  __host__ __device__ static constexpr int k(int rho) {
+    if (B == 1) return (rho >= 5 && rho <= 9) ? rho : (rho >= 10 && rho <= 14) ? rho - 5 : (rho <= 4) ? rho + 5 : 9;
+    if (B == 2) {
+      const int l = rho & 7, o = 2 * l;
+      return (l >= 2 && l <= 4) ? o : (l >= 5) ? o - 6 : o + 4;
+    }
+    return 10 - B;
+  }
+  __host__ __device__ static constexpr float off(int rho) { return (float)(1 << (10 - k(rho))); }
+};
+
+template <int B>
+__host__ __device__ __forceinline__ void load_piece(const uint8_t* p, uint32_t (&w)[B]) {
+  if constexpr (B % 4 == 0) {
+#pragma unroll
+    for (int i = 0; i < B / 4; ++i) {
+      const uint4 v = reinterpret_cast<const uint4*>(p)[i];
+      w[4 * i + 0] = v.x;
+      w[4 * i + 1] = v.y;
+      w[4 * i + 2] = v.z;
+      w[4 * i + 3] = v.w;
+    }
+  } else if constexpr (B == 2) {
+    const uint2 v = *reinterpret_cast<const uint2*>(p);
+    w[0] = v.x;
+    w[1] = v.y;
+  } else {
+#pragma unroll
+    for (int i = 0; i < B; ++i) w[i] = reinterpret_cast<const uint32_t*>(p)[i];
+  }
+}
+
+template <int B>
+__host__ __device__ __forceinline__ void unpack_piece(const uint32_t (&w)[B], uint32_t (&o)[16]) {
+  if constexpr (B == 1) {
+    const uint32_t x = w[0], xr5 = x >> 5, xl5 = x << 5, xr6 = x >> 6;
+#pragma unroll
+    for (int rho = 0; rho < 16; ++rho) {
+      const int k = Window<1>::k(rho);
+      const uint32_t t = (rho >= 5 && rho <= 9) ? x : (rho >= 10 && rho <= 14) ? xr5 : (rho <= 4) ? xl5 : xr6;
+      o[rho] = (t & pair_mask(1, k)) | magic2(k);
+    }
+  } else if constexpr (B == 2) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const uint32_t x = w[half], xr6 = x >> 6, xl4 = x << 4;
+#pragma unroll
+      for (int l = 0; l < 8; ++l) {
+        const int rho = 8 * half + l;
+        const int k = Window<2>::k(rho);
+        const uint32_t t = (l >= 2 && l <= 4) ? x : (l >= 5) ? xr6 : xl4;
+        o[rho] = (t & pair_mask(2, k)) | magic2(k);
+      }
+    }
+  } else {
+    constexpr int k = 10 - B;
+#pragma unroll
+    for (int rho = 0; rho < 16; ++rho) {
+      const int x = rho * B, wi = x >> 4, off = x & 15;
+      if (off + B <= 16) {
+        const uint32_t t = (off >= k) ? (w[wi] >> (off - k)) : (w[wi] << (k - off));
+        o[rho] = (t & pair_mask(B, k)) | magic2(k);
+      } else {
+        const int nlo = 16 - off;
+        const uint32_t lo = w[wi] >> (off - k);
+        const uint32_t hi = w[wi + 1] << (k + nlo);
+        o[rho] = (lo & pair_mask(nlo, k)) | (hi & pair_mask(B - nlo, k + nlo)) | magic2(k);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// parameter block access
+// ---------------------------------------------------------------------------------------
+__device__ __forceinline__ const HeadEntry* head_table(const unsigned char* block) {
+  const BlockHeader* h = reinterpret_cast<const BlockHeader*>(block);
+  return reinterpret_cast<const HeadEntry*>(block + h->heads_off);
+}
+__device__ __forceinline__ const float* param_pool(const unsigned char* block) {
+  const BlockHeader* h = reinterpret_cast<const BlockHeader*>(block);
+  return reinterpret_cast<const float*>(block + h->pool_off);
+}
+
+// Byte address of code row `row` of sequence `seq` inside a head region.
+__device__ __forceinline__ uint64_t row_offset(uint64_t region, uint32_t row_bytes, int seq, int row,
+                                               const int* page_table, int pages_per_seq, int rows_per_seq) {
+  long long slot;
+  if (page_table)
+    slot = 2LL * page_table[(long long)seq * pages_per_seq + (row >> 1)] + (row & 1);
+  else
+    slot = (long long)seq * rows_per_seq + row;
+  return region + (uint64_t)slot * row_bytes;
+}
+
+}  // namespace cobra
