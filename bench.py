@@ -1,0 +1,408 @@
+#!/usr/bin/env python
+"""Decode-step benchmark of the KV-COBRA hot path on GB300.
+
+Workload (default): the Llama-3-8B-shaped compressed cache - 32 layers x 8 KV heads x
+head_dim 128, 32 query heads, batch 8 x 32768-token contexts, K and V allocated separately
+at 1 bpd (KL weights for K).  One step = append-compress the new token's K and V for every
+(layer, kv head, sequence) into the packed cache, then decode attention for one query per
+query head across all layers (query projection, rank-space scan over the packed codes,
+combine + back-projection).
+
+Reported: effective HBM GB/s over the packed cache (packed bytes a step reads / step time),
+the scan kernel's roofline fraction against the measured HBM copy bandwidth, an end-to-end
+number through host buffers, and the fp64 oracle timed on the host cores on a bounded
+sample.  Under torchrun each rank runs its own replica (weak scaling, no collective on the
+data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode-attn effective HBM GB/s over packed cache (% of peak); compress tok/s"
+FALLBACK_HBM_GBS = 6800.0
+PROFILE = os.path.join(ROOT, "profiles", "decode_scan_llama3_8b.txt")
+SCAN_SOURCES = ["paper_2609_24298_gb300/csrc/decode.cuh", "paper_2609_24298_gb300/csrc/common.cuh"]
+CFG = 2
+SAMPLE_R, SAMPLE_B = 64, 2  # (r, b) of the oracle sample heads: the most common point at 1 bpd
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="cobra", choices=["cobra", "reference"])
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle sample budget for cpu_baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None, help="fewer layers (profiling runs only)")
+    return ap.parse_args()
+
+
+def scan_source_hash() -> str:
+    h = hashlib.sha256()
+    for p in SCAN_SOURCES:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per scan launch from the committed ncu summary, if it was taken on the
+    current kernel source (else None)."""
+    try:
+        txt = open(PROFILE).read()
+    except OSError:
+        return None
+    m1 = re.search(r"traffic_bytes_per_launch\s*=\s*([0-9.eE+]+)", txt)
+    m2 = re.search(r"kernel_source_sha\s*=\s*([0-9a-f]+)", txt)
+    if not m1 or not m2 or m2.group(1) != scan_source_hash():
+        return None
+    return float(m1.group(1))
+
+
+def hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------------------
+# fp64 oracle on the host cores (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------------------
+class OracleSample:
+    """One (sequence, layer, kv head) group of the workload run by the oracle: decode
+    attention over T tokens of packed codes plus the append-compress of the new token, with
+    K and V at (r, b) = (SAMPLE_R, SAMPLE_B).  Setup (calibration, compressing the context) is
+    untimed."""
+
+    def __init__(self, head: int, T: int, group: int):
+        from oracle import calibrate as ocal
+        from oracle import compress as ocomp
+        from paper_2609_24298_gb300 import synth
+
+        spec = synth.CONFIGS[CFG]
+        self.params, self.codes, self.new = [], [], []
+        for side in (0, 1):
+            src = synth.HeadSource(CFG, 0, head, side, spec["alpha"])
+            cal = ocal.calibrate_head(src.calibration(512))
+            p = ocal.head_params(cal, SAMPLE_R, SAMPLE_B, synth.hadamard_signs(*src.key))
+            x = src.tokens(T)
+            _, c = ocomp.compress(x[:-1], p["W"], p["mu"], p["delta"], SAMPLE_B)
+            self.params.append(p)
+            self.codes.append(c)
+            self.new.append(x[-1:])
+        self.q = synth.decode_queries(CFG, 0, head, 1, group)[0].astype(np.float64)
+        self.bytes = 2 * ((T * SAMPLE_R * SAMPLE_B + 7) // 8 + 15) // 16 * 16
+
+    def step(self):
+        from oracle import attention as oatt
+        from oracle import compress as ocomp
+
+        codes = []
+        for side in (0, 1):
+            p = self.params[side]
+            _, c = ocomp.compress(self.new[side], p["W"], p["mu"], p["delta"], SAMPLE_B)
+            codes.append(np.concatenate([self.codes[side], c]))
+        return oatt.decode(self.q, codes[0], codes[1], self.params[0], self.params[1])
+
+
+def oracle_rate(seconds: float, T: int, group: int):
+    """Packed bytes per second the oracle processes, timed over about `seconds` of work."""
+    samples = [OracleSample(h, T, group) for h in range(2)]
+    done, nbytes, t0 = 0, 0, time.perf_counter()
+    while True:
+        s = samples[done % len(samples)]
+        s.step()
+        nbytes += s.bytes
+        done += 1
+        el = time.perf_counter() - t0
+        if el >= seconds and done >= 2:
+            break
+    return nbytes / el / 1e9, done, el
+
+
+def cores_used():
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(k, "").isdigit():
+            return int(os.environ[k])
+    return os.cpu_count()
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_24298_gb300 import synth
+
+    spec = synth.CONFIGS[CFG]
+    T, group = spec["tokens"], spec["q_heads"] // spec["kv_heads"]
+    sample = OracleSample(0, T, group)
+    for _ in range(args.warmup):
+        sample.step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        sample.step()
+    el = time.perf_counter() - t0
+    gbs = sample.bytes * args.steps / el / 1e9
+    desc = (f"one (seq, layer, kv-head) group per step: decode over {T} tokens with K and V at r={SAMPLE_R}, "
+            f"b={SAMPLE_B} + append-compress of the new token (fp64 numpy)")
+    out = {"metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": args.gpus, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+           "config": workload_config(spec),
+           "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores_used(), "kind": "oracle", "sample": desc},
+           "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def workload_config(spec):
+    return {"workload": "llama3-8b-shaped decode step: 32 layers x 8 kv heads (GQA 4, head_dim 128) x batch 8 x "
+                        "32768-token context, K and V at 1 bpd",
+            "layers": spec["layers"], "kv_heads": spec["kv_heads"], "q_heads": spec["q_heads"],
+            "batch": spec["seqs"], "context": spec["tokens"], "bpd": spec["bpd"],
+            "step": "append K+V of 1 token per (layer, kv head, seq) + decode attention for all layers",
+            "l2": "inputs larger than L2 (packed cache of about 2 GiB re-read every step)"}
+
+
+# ---------------------------------------------------------------------------------------
+# the CUDA path
+# ---------------------------------------------------------------------------------------
+def run_cobra(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_24298_gb300 import cobra, pipeline, synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    spec = synth.CONFIGS[CFG]
+    L, H, S, T = spec["layers"], spec["kv_heads"], spec["seqs"], spec["tokens"]
+    if args.layers:
+        L = args.layers
+    G = spec["q_heads"] // H
+    Hq = H * G
+    cobra.lib()
+
+    # cpu baseline first, before any GPU work (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        gbs, n, el = oracle_rate(args.cpu_seconds, T, G)
+        cpu = {"value": gbs, "unit": "GB/s", "cores": cores_used(), "kind": "oracle",
+               "sample": f"{n} (seq, layer, kv-head) decode steps over {T} tokens with K and V at r={SAMPLE_R}, "
+                         f"b={SAMPLE_B} incl. append-compress ({el:.1f} s of fp64 numpy)"}
+
+    hp, srcs = pipeline.build_params(CFG, L, spec["bpd"], joint=False)
+    rows = -(-T // 128)
+    wl = pipeline.Workload(cfg=CFG, layers=L, kv=H, group=G, seqs=S, tokens=np.full(S, T - 1, np.int64),
+                           bpd=spec["bpd"], joint=False, rows_per_seq=rows)
+    wl.dev = pipeline.DeviceParams(hp, S * rows, device=dev)
+    pipeline.fill_cache(wl, srcs, device=dev)
+    wl.tokens = np.full(S, T, np.int64)
+    desc, ws, info = pipeline.decode_setup(wl, device=dev)
+    nbytes_ws = ws.numel()
+    stream = torch.cuda.current_stream()
+
+    # per-step inputs: the new token's K and V for every (layer, kv head, seq); the queries
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(2609 + rank)
+    xk = torch.randn((L, S, H, 128), generator=gen, device=dev).to(torch.bfloat16)
+    xv = torch.randn((L, S, H, 128), generator=gen, device=dev).to(torch.bfloat16)
+    q = torch.randn((L, S, Hq, 128), generator=gen, device=dev).to(torch.bfloat16)
+    out = torch.empty((L, S, Hq, 128), dtype=torch.float32, device=dev)
+    pos = torch.full((S,), T - 1, dtype=torch.int32, device=dev)
+    lens = torch.full((S,), T, dtype=torch.int32, device=dev)
+    adesc = [cobra.compress_desc(head0=side * L * H, layer_stride=H, n_layers=L, n_kv_heads=H, side=side, n_seqs=S,
+                                 rows_per_seq=rows, x_stride_layer=S * H * 128, x_stride_seq=H * 128, x_stride_tok=0,
+                                 x_stride_head=128) for side in (0, 1)]
+    block, cache = wl.dev.block, wl.dev.cache
+
+    def step(ev_scan0=None, ev_scan1=None):
+        cobra.cobra_append(block, adesc[0], xk, pos, cache, None, stream)
+        cobra.cobra_append(block, adesc[1], xv, pos, cache, None, stream)
+        cobra.cobra_decode_qproj(block, desc, info, q, ws, nbytes_ws, stream)
+        if ev_scan0 is not None:
+            ev_scan0.record(stream)
+        cobra.cobra_decode_scan(block, desc, info, cache, lens, None, ws, nbytes_ws, stream)
+        if ev_scan1 is not None:
+            ev_scan1.record(stream)
+        cobra.cobra_decode_combine(block, desc, info, lens, out, ws, nbytes_ws, stream)
+
+    launches_per_step = 5
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    st = cobra.cobra_check(stream)
+    if st != cobra.COBRA_OK:
+        raise RuntimeError(f"device status {st} after warm-up")
+
+    # timed region: the whole steps, and the scan kernel alone (events on the launch stream)
+    K = args.steps
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    t_start.record(stream)
+    for k in range(K):
+        step(ev[k][0], ev[k][1])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    scan_ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    st = cobra.cobra_check(stream)
+    if st != cobra.COBRA_OK:
+        raise RuntimeError(f"device status {st} after the timed region")
+
+    bytes_step = pipeline.packed_bytes_read(wl)
+    value = bytes_step * K * world / (total_ms * 1e-3) / 1e9
+
+    # end to end through the public API: pinned host inputs in, host output out, every step
+    hk = torch.empty_like(xk, device="cpu").pin_memory()
+    hv = torch.empty_like(xv, device="cpu").pin_memory()
+    hq = torch.empty_like(q, device="cpu").pin_memory()
+    hout = torch.empty_like(out, device="cpu").pin_memory()
+    hk.copy_(xk.cpu())
+    hv.copy_(xv.cpu())
+    hq.copy_(q.cpu())
+    Ke = max(10, K // 4)
+
+    def e2e_step():
+        xk.copy_(hk, non_blocking=True)
+        xv.copy_(hv, non_blocking=True)
+        q.copy_(hq, non_blocking=True)
+        cobra.cobra_append(block, adesc[0], xk, pos, cache, None, stream)
+        cobra.cobra_append(block, adesc[1], xv, pos, cache, None, stream)
+        cobra.cobra_decode_attn(block, desc, info, q, cache, lens, None, out, ws, nbytes_ws, stream)
+        hout.copy_(out, non_blocking=True)
+
+    for _ in range(5):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(Ke):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / Ke
+    if world > 1:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    h2d = (xk.numel() + xv.numel() + q.numel()) * 2
+    d2h = out.numel() * 4
+
+    peak, peak_kind = hbm_peak()
+    achieved = bytes_step / (scan_ms * 1e-3) / 1e9
+    traffic = profiled_traffic()
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": K, "warmup": args.warmup,
+            "ms_per_step": total_ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "fp16-mma/fp32-acc on 1-8 bit codes", "data": "synthetic", "impl": "cobra",
+            "config": workload_config(spec) | {"parallelism": f"replicas x{world}", "layers": L,
+                                               "packed_bytes_per_step": bytes_step},
+            "roofline": {"bound": "hbm", "kernel": "decode_kernel (rank-space scan)", "achieved": achieved,
+                         "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": traffic, "scan_ms": scan_ms,
+                         "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
+            "cpu_baseline": cpu,
+            "e2e": {"value": bytes_step * world / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "gpu_launches": launches_per_step * K,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_cobra(args)
+
+
+if __name__ == "__main__":
+    main()
