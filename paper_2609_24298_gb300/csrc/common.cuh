@@ -87,6 +87,12 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
   asm("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
   return y;
 }
+// 2^x with the SFU's approximate exponential (flush-to-zero; relative error about 2^-22)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 __device__ __forceinline__ uint32_t pack_f16(float lo_col, float hi_col) {
   __half2 h = __floats2half2_rn(lo_col, hi_col);  // .x -> low 16 bits
   return *reinterpret_cast<uint32_t*>(&h);
@@ -142,43 +148,48 @@ __host__ __device__ __forceinline__ void load_piece(const uint8_t* p, uint32_t (
   }
 }
 
+// One register: codes (rho, 0) and (rho, 1) of the piece held in w.  rho is a compile-time
+// constant wherever this is called from an unrolled loop.
 template <int B>
-__host__ __device__ __forceinline__ void unpack_piece(const uint32_t (&w)[B], uint32_t (&o)[16]) {
+__host__ __device__ __forceinline__ uint32_t unpack_reg(const uint32_t (&w)[B], int rho) {
   if constexpr (B == 1) {
-    const uint32_t x = w[0], xr5 = x >> 5, xl5 = x << 5, xr6 = x >> 6;
-#pragma unroll
-    for (int rho = 0; rho < 16; ++rho) {
-      const int k = Window<1>::k(rho);
-      const uint32_t t = (rho >= 5 && rho <= 9) ? x : (rho >= 10 && rho <= 14) ? xr5 : (rho <= 4) ? xl5 : xr6;
-      o[rho] = (t & pair_mask(1, k)) | magic2(k);
-    }
+    const int k = Window<1>::k(rho);
+    const uint32_t x = w[0];
+    const uint32_t t = (rho >= 5 && rho <= 9) ? x : (rho >= 10 && rho <= 14) ? (x >> 5) : (rho <= 4) ? (x << 5) : (x >> 6);
+    return (t & pair_mask(1, k)) | magic2(k);
   } else if constexpr (B == 2) {
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const uint32_t x = w[half], xr6 = x >> 6, xl4 = x << 4;
-#pragma unroll
-      for (int l = 0; l < 8; ++l) {
-        const int rho = 8 * half + l;
-        const int k = Window<2>::k(rho);
-        const uint32_t t = (l >= 2 && l <= 4) ? x : (l >= 5) ? xr6 : xl4;
-        o[rho] = (t & pair_mask(2, k)) | magic2(k);
-      }
-    }
+    const int l = rho & 7, k = Window<2>::k(rho);
+    const uint32_t x = w[rho >> 3];
+    const uint32_t t = (l >= 2 && l <= 4) ? x : (l >= 5) ? (x >> 6) : (x << 4);
+    return (t & pair_mask(2, k)) | magic2(k);
   } else {
     constexpr int k = 10 - B;
-#pragma unroll
-    for (int rho = 0; rho < 16; ++rho) {
-      const int x = rho * B, wi = x >> 4, off = x & 15;
-      if (off + B <= 16) {
-        const uint32_t t = (off >= k) ? (w[wi] >> (off - k)) : (w[wi] << (k - off));
-        o[rho] = (t & pair_mask(B, k)) | magic2(k);
-      } else {
-        const int nlo = 16 - off;
-        const uint32_t lo = w[wi] >> (off - k);
-        const uint32_t hi = w[wi + 1] << (k + nlo);
-        o[rho] = (lo & pair_mask(nlo, k)) | (hi & pair_mask(B - nlo, k + nlo)) | magic2(k);
-      }
+    const int x = rho * B, wi = x >> 4, off = x & 15;
+    if (off + B <= 16) {
+      const uint32_t t = (off >= k) ? (w[wi] >> (off - k)) : (w[wi] << (k - off));
+      return (t & pair_mask(B, k)) | magic2(k);
     }
+    const int nlo = 16 - off;
+    const uint32_t lo = w[wi] >> (off - k);
+    const uint32_t hi = w[(wi + 1) < B ? wi + 1 : wi] << (k + nlo);
+    return (lo & pair_mask(nlo, k)) | (hi & pair_mask(B - nlo, k + nlo)) | magic2(k);
+  }
+}
+
+template <int B>
+__host__ __device__ __forceinline__ void unpack_piece(const uint32_t (&w)[B], uint32_t (&o)[16]) {
+#pragma unroll
+  for (int rho = 0; rho < 16; ++rho) o[rho] = unpack_reg<B>(w, rho);
+}
+
+// Words of the piece at p, or zeros when the strip does not exist.
+template <int B>
+__device__ __forceinline__ void load_piece_or_zero(const uint8_t* p, bool valid, uint32_t (&w)[B]) {
+  if (valid) {
+    load_piece<B>(p, w);
+  } else {
+#pragma unroll
+    for (int i = 0; i < B; ++i) w[i] = 0u;
   }
 }
 

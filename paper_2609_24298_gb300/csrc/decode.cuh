@@ -20,6 +20,7 @@
 namespace cobra {
 
 constexpr int kDecodeWarps = 4;
+constexpr int kMaxStages = 8;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 
 struct DecodeArgs {
@@ -32,7 +33,7 @@ struct DecodeArgs {
   unsigned char* ws;
   long long q_sl, q_ss, o_sl, o_ss;
   int rows_per_seq, pages_per_seq;
-  int stage_bytes, nstage;
+  int ring_bytes;  // per-warp staging ring (>= 2 of the largest code rows, multiple of 128)
 };
 
 // ---------------------------------------------------------------------------------------
@@ -133,19 +134,24 @@ __global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
 
 // ---------------------------------------------------------------------------------------
 // a5 + a6: chunked rank-space scan
+//
+// Per warp: running max m, sum l and offset correction c per query head in registers; the
+// rank-space value accumulators O[nt][mu] (lane-owned float4 of the MMA C fragment) live in
+// the warp's shared memory and are rescaled only when the running max moves.  Loops over
+// k-tiles (K side) and channel tiles (V side) stay rolled to keep each (b_K, b_V) variant's
+// code small; only the 8 token tiles of a row are unrolled.
 // ---------------------------------------------------------------------------------------
 template <int G>
 struct WarpState {
   static constexpr int NT = G / 4;
   float m[NT], l[NT], c[NT];
-  float o[NT][8][4];
 };
 
-// K side: scores of one code row for the lane's query heads.  Returns scores in s[8][NT][2]
+// K side: scores of one code row for the lane's query heads, s[8][NT][2]
 // (token t0 = 16 tau + lane/4 in [..][..][0], t1 = t0 + 8 in [..][..][1]), log2 units.
 template <int G, int B>
-__device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const uint2* bfrag, const float* qsum,
-                                             float qscale, float (&s)[8][G / 4][2]) {
+__device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const uint2* bfrag,
+                                             const float (&qg)[G / 4], float qscale, float (&s)[8][G / 4][2]) {
   constexpr int NT = G / 4;
   const int lane = threadIdx.x & 31;
   float acc[8][NT][4];
@@ -155,138 +161,132 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
     for (int nt = 0; nt < NT; ++nt) acc[t][nt][0] = acc[t][nt][1] = acc[t][nt][2] = acc[t][nt][3] = 0.f;
   const int P = rk >> 1;
   const int nk = (P + 7) >> 3;
+  const int pc = lane >> 2;
+#pragma unroll 1
+  for (int kap = 0; kap < nk; ++kap) {
+    // channels past r (a partial last k-tile) multiply q~ = 0, so their operand values only
+    // need to be finite; the words are zeroed rather than read past the row
+    const int sA = 8 * kap + (lane & 3), sB = sA + 4;
+    uint32_t wa[B], wb[B];
+    load_piece_or_zero<B>(stage + sA * 32 * B + pc * 4 * B, sA < P, wa);
+    load_piece_or_zero<B>(stage + sB * 32 * B + pc * 4 * B, sB < P, wb);
+    uint2 bf[NT];
 #pragma unroll
-  for (int kap = 0; kap < 8; ++kap) {
-    if (kap < nk) {
-      const int sA = 8 * kap + (lane & 3), sB = sA + 4, pc = lane >> 2;
-      uint32_t pa[16], pb[16];
-      if (sA < P) {
-        uint32_t w[B];
-        load_piece<B>(stage + sA * 32 * B + pc * 4 * B, w);
-        unpack_piece<B>(w, pa);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) pa[i] = 0u;
-      }
-      if (sB < P) {
-        uint32_t w[B];
-        load_piece<B>(stage + sB * 32 * B + pc * 4 * B, w);
-        unpack_piece<B>(w, pb);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 16; ++i) pb[i] = 0u;
-      }
-      uint2 bf[NT];
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) bf[nt] = bfrag[(kap * 2 + nt) * 32 + lane];
-#pragma unroll
-      for (int t = 0; t < 8; ++t)
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-          mma_f16(acc[t][nt], pa[2 * t], pa[2 * t + 1], pb[2 * t], pb[2 * t + 1], bf[nt].x, bf[nt].y);
-    }
-  }
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    const float qg = qsum[4 * nt + (lane & 3)];
+    for (int nt = 0; nt < NT; ++nt) bf[nt] = bfrag[(kap * 2 + nt) * 32 + lane];
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
-      s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1] - Window<B>::off(2 * t) * qg) * qscale;
-      s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3] - Window<B>::off(2 * t + 1) * qg) * qscale;
+      const uint32_t a0 = unpack_reg<B>(wa, 2 * t), a1 = unpack_reg<B>(wa, 2 * t + 1);
+      const uint32_t a2 = unpack_reg<B>(wb, 2 * t), a3 = unpack_reg<B>(wb, 2 * t + 1);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) mma_f16(acc[t][nt], a0, a1, a2, a3, bf[nt].x, bf[nt].y);
+    }
+  }
+  // b >= 3 uses one window for every register, so the offset adds the same constant to every
+  // token's score and softmax ignores it; b = 1, 2 mix windows and need the per-token term
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      if constexpr (B <= 2) {
+        s[t][nt][0] = fmaf(acc[t][nt][0] + acc[t][nt][1], qscale, -Window<B>::off(2 * t) * qg[nt]);
+        s[t][nt][1] = fmaf(acc[t][nt][2] + acc[t][nt][3], qscale, -Window<B>::off(2 * t + 1) * qg[nt]);
+      } else {
+        s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1]) * qscale;
+        s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3]) * qscale;
+      }
     }
   }
 }
 
-// V side: accumulate one code row into o (rank space) and the offset correction into c.
+// V side: add one code row's rank-space contribution into the shared-memory accumulators.
 template <int G, int B>
 __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, const uint32_t (&bv)[8][G / 4][2],
-                                                 const float (&p)[8][G / 4][2], WarpState<G>& st) {
+                                                 float4* osm) {
   constexpr int NT = G / 4;
   const int lane = threadIdx.x & 31;
   const int P = rv >> 1;
   const int nmu = (P + 7) >> 3;
+  const int pc = lane & 7;
+#pragma unroll 1
+  for (int mu = 0; mu < nmu; ++mu) {
+    // rows for channels past r are never written out, so their operand values only need to
+    // be finite
+    const int sA = 8 * mu + (lane >> 3), sB = sA + 4;
+    uint32_t wa[B], wb[B];
+    load_piece_or_zero<B>(stage + sA * 32 * B + pc * 4 * B, sA < P, wa);
+    load_piece_or_zero<B>(stage + sB * 32 * B + pc * 4 * B, sB < P, wb);
+    float d[NT][2][4];
 #pragma unroll
-  for (int mu = 0; mu < 8; ++mu) {
-    if (mu < nmu) {
-      const int sA = 8 * mu + (lane >> 3), sB = sA + 4, pc = lane & 7;
-      uint32_t pa[16], pb[16];
-      if (sA < P) {
-        uint32_t w[B];
-        load_piece<B>(stage + sA * 32 * B + pc * 4 * B, w);
-        unpack_piece<B>(w, pa);
-      } else {
+    for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-        for (int i = 0; i < 16; ++i) pa[i] = 0u;
-      }
-      if (sB < P) {
-        uint32_t w[B];
-        load_piece<B>(stage + sB * 32 * B + pc * 4 * B, w);
-        unpack_piece<B>(w, pb);
-      } else {
+      for (int u = 0; u < 2; ++u) d[nt][u][0] = d[nt][u][1] = d[nt][u][2] = d[nt][u][3] = 0.f;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) pb[i] = 0u;
-      }
+    for (int t = 0; t < 8; ++t) {
+      const uint32_t a0 = unpack_reg<B>(wa, 2 * t), a1 = unpack_reg<B>(wb, 2 * t);
+      const uint32_t a2 = unpack_reg<B>(wa, 2 * t + 1), a3 = unpack_reg<B>(wb, 2 * t + 1);
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        float d[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int t = 0; t < 8; ++t) mma_f16(d, pa[2 * t], pb[2 * t], pa[2 * t + 1], pb[2 * t + 1], bv[t][nt][0], bv[t][nt][1]);
-        st.o[nt][mu][0] += d[0];
-        st.o[nt][mu][1] += d[1];
-        st.o[nt][mu][2] += d[2];
-        st.o[nt][mu][3] += d[3];
-      }
+      for (int nt = 0; nt < NT; ++nt) mma_f16(d[nt][t & 1], a0, a1, a2, a3, bv[t][nt][0], bv[t][nt][1]);
     }
-  }
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    float c = 0.f;
-#pragma unroll
-    for (int t = 0; t < 8; ++t) c += p[t][nt][0] * Window<B>::off(2 * t) + p[t][nt][1] * Window<B>::off(2 * t + 1);
-    st.c[nt] += c;
+    for (int nt = 0; nt < NT; ++nt) {
+      float4* o = osm + (nt * 8 + mu) * 32 + lane;
+      float4 v = *o;
+      v.x += d[nt][0][0] + d[nt][1][0];
+      v.y += d[nt][0][1] + d[nt][1][1];
+      v.z += d[nt][0][2] + d[nt][1][2];
+      v.w += d[nt][0][3] + d[nt][1][3];
+      *o = v;
+    }
   }
 }
 
 template <int G>
-__device__ __forceinline__ void k_row_dispatch(int b, const uint8_t* stage, int rk, const uint2* bfrag, const float* qsum,
-                                               float qscale, float (&s)[8][G / 4][2]) {
+__device__ __forceinline__ void k_row_dispatch(int b, const uint8_t* stage, int rk, const uint2* bfrag,
+                                               const float (&qg)[G / 4], float qscale, float (&s)[8][G / 4][2]) {
   switch (b) {
-    case 1: k_row_scores<G, 1>(stage, rk, bfrag, qsum, qscale, s); break;
-    case 2: k_row_scores<G, 2>(stage, rk, bfrag, qsum, qscale, s); break;
-    case 3: k_row_scores<G, 3>(stage, rk, bfrag, qsum, qscale, s); break;
-    case 4: k_row_scores<G, 4>(stage, rk, bfrag, qsum, qscale, s); break;
-    case 5: k_row_scores<G, 5>(stage, rk, bfrag, qsum, qscale, s); break;
-    case 6: k_row_scores<G, 6>(stage, rk, bfrag, qsum, qscale, s); break;
-    case 7: k_row_scores<G, 7>(stage, rk, bfrag, qsum, qscale, s); break;
-    default: k_row_scores<G, 8>(stage, rk, bfrag, qsum, qscale, s); break;
+    case 1: k_row_scores<G, 1>(stage, rk, bfrag, qg, qscale, s); break;
+    case 2: k_row_scores<G, 2>(stage, rk, bfrag, qg, qscale, s); break;
+    case 3: k_row_scores<G, 3>(stage, rk, bfrag, qg, qscale, s); break;
+    case 4: k_row_scores<G, 4>(stage, rk, bfrag, qg, qscale, s); break;
+    case 5: k_row_scores<G, 5>(stage, rk, bfrag, qg, qscale, s); break;
+    case 6: k_row_scores<G, 6>(stage, rk, bfrag, qg, qscale, s); break;
+    case 7: k_row_scores<G, 7>(stage, rk, bfrag, qg, qscale, s); break;
+    default: k_row_scores<G, 8>(stage, rk, bfrag, qg, qscale, s); break;
   }
 }
 
 template <int G>
 __device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int rv, const uint32_t (&bv)[8][G / 4][2],
-                                               const float (&p)[8][G / 4][2], WarpState<G>& st) {
+                                               float4* osm) {
   switch (b) {
-    case 1: v_row_accumulate<G, 1>(stage, rv, bv, p, st); break;
-    case 2: v_row_accumulate<G, 2>(stage, rv, bv, p, st); break;
-    case 3: v_row_accumulate<G, 3>(stage, rv, bv, p, st); break;
-    case 4: v_row_accumulate<G, 4>(stage, rv, bv, p, st); break;
-    case 5: v_row_accumulate<G, 5>(stage, rv, bv, p, st); break;
-    case 6: v_row_accumulate<G, 6>(stage, rv, bv, p, st); break;
-    case 7: v_row_accumulate<G, 7>(stage, rv, bv, p, st); break;
-    default: v_row_accumulate<G, 8>(stage, rv, bv, p, st); break;
+    case 1: v_row_accumulate<G, 1>(stage, rv, bv, osm); break;
+    case 2: v_row_accumulate<G, 2>(stage, rv, bv, osm); break;
+    case 3: v_row_accumulate<G, 3>(stage, rv, bv, osm); break;
+    case 4: v_row_accumulate<G, 4>(stage, rv, bv, osm); break;
+    case 5: v_row_accumulate<G, 5>(stage, rv, bv, osm); break;
+    case 6: v_row_accumulate<G, 6>(stage, rv, bv, osm); break;
+    case 7: v_row_accumulate<G, 7>(stage, rv, bv, osm); break;
+    default: v_row_accumulate<G, 8>(stage, rv, bv, osm); break;
   }
 }
 
 template <int G>
-__global__ void __launch_bounds__(kDecodeWarps * 32) decode_kernel(DecodeArgs a) {
+__device__ __forceinline__ size_t decode_osm_bytes() {
+  return (size_t)(G / 4) * 8 * 32 * sizeof(float4);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs a) {
   constexpr int NT = G / 4;
   extern __shared__ __align__(128) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nstage = a.nstage, stage_bytes = a.stage_bytes;
-  uint8_t* ring = smem + (size_t)warp * nstage * stage_bytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)kDecodeWarps * nstage * stage_bytes) + warp * nstage;
+  const int ring_bytes = a.ring_bytes;
+  const size_t warp_bytes = (size_t)ring_bytes + decode_osm_bytes<G>();
+  uint8_t* ring = smem + (size_t)warp * warp_bytes;
+  float4* osm = reinterpret_cast<float4*>(ring + ring_bytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)kDecodeWarps * warp_bytes) + warp * kMaxStages;
   if (lane == 0) {
-    for (int i = 0; i < nstage; ++i) mbar_init(smem_addr(&bars[i]), 1);
+    for (int i = 0; i < kMaxStages; ++i) mbar_init(smem_addr(&bars[i]), 1);
     fence_mbar_init();
   }
   __syncwarp();
@@ -298,30 +298,28 @@ __global__ void __launch_bounds__(kDecodeWarps * 32) decode_kernel(DecodeArgs a)
   float* parts = reinterpret_cast<float*>(a.ws + wh->part_off);
   const int n_items = wh->n_items;
   const int gstride = wh->g_stride, pstride = wh->part_stride;
-  uint32_t phase_bits = 0;  // parity of the next wait per stage
+  uint32_t phase_bits = 0;  // parity of the next wait per barrier
   bool failed = false;
   int outstanding = 0;      // loads issued but not yet waited for (stages are used in order)
   int next_wait_stage = 0;
+  int nstage = 2, stage_bytes = ring_bytes / 2;
 
   for (int item = blockIdx.x * kDecodeWarps + warp; item < n_items && !failed; item += gridDim.x * kDecodeWarps) {
     const WsItem it = items[item];
     const WsGroup gr = groups[it.group];
-    const HeadEntry hk = heads[gr.k_head], hv = heads[gr.v_head];
+    const int kr = heads[gr.k_head].r, kb = heads[gr.k_head].b, vr = heads[gr.v_head].r, vb = heads[gr.v_head].b;
+    const uint64_t koff = heads[gr.k_head].cache_off, voff = heads[gr.v_head].cache_off;
     const int T = a.seq_lens[gr.seq];
     const int rows_valid = (T + kRowTokens - 1) / kRowTokens;
     const int row0 = it.row_begin, row1 = min(it.row_end, rows_valid);
     float* part = parts + (size_t)item * pstride;
-    WarpState<G> st;
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      st.m[nt] = -INFINITY;
-      st.l[nt] = 0.f;
-      st.c[nt] = 0.f;
-#pragma unroll
-      for (int mu = 0; mu < 8; ++mu) st.o[nt][mu][0] = st.o[nt][mu][1] = st.o[nt][mu][2] = st.o[nt][mu][3] = 0.f;
-    }
-    const uint32_t rbk = hk.r > 0 ? 16u * hk.r * hk.b : 0u, rbv = hv.r > 0 ? 16u * hv.r * hv.b : 0u;
-    if (rbk > (uint32_t)stage_bytes || rbv > (uint32_t)stage_bytes) {
+    const uint32_t rbk = kr > 0 ? 16u * kr * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
+    // this item's stages: as many buffers of its largest row as the ring holds (every load of
+    // the previous item has been consumed, so the ring is free)
+    stage_bytes = (int)((max(max(rbk, rbv), 16u) + 127u) & ~127u);
+    nstage = min(kMaxStages, ring_bytes / stage_bytes);
+    next_wait_stage = 0;
+    if (nstage < 2) {
       // a row that does not fit the staging buffer is never copied; report and leave an
       // empty chunk (m = -inf, l = 0)
       if (lane == 0) atomicOr(&g_status, 2u);
@@ -331,68 +329,84 @@ __global__ void __launch_bounds__(kDecodeWarps * 32) decode_kernel(DecodeArgs a)
       }
       continue;
     }
+    WarpState<G> st;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      st.m[nt] = -INFINITY;
+      st.l[nt] = 0.f;
+      st.c[nt] = 0.f;
+    }
+    const int nmu = ((vr >> 1) + 7) >> 3;
+    // V offsets: b >= 3 has one window, so the correction is 2^b * l (added at the end);
+    // b = 1, 2 need the per-token sum
+    const bool vsmall = vr > 0 && vb <= 2;
+    for (int k = 0; k < NT * nmu; ++k) {
+      const int nt = k / nmu, mu = k % nmu;
+      osm[(nt * 8 + mu) * 32 + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     const int loads_per_row = (rbk ? 1 : 0) + (rbv ? 1 : 0);
     const int n_loads = row1 > row0 ? (row1 - row0) * loads_per_row : 0;
     const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
     const float* qhdr = reinterpret_cast<const float*>(qt);
     const uint2* bfrag = reinterpret_cast<const uint2*>(qt + kQtHeaderBytes);
-    float qsum[G];
+    float qg[NT];
 #pragma unroll
-    for (int g = 0; g < G; ++g) qsum[g] = qhdr[g];
+    for (int nt = 0; nt < NT; ++nt) qg[nt] = qhdr[4 * nt + (lane & 3)] * qhdr[8];
     const float qscale = qhdr[8];
 
     // load n of this item -> (row, side)
-    auto load_src = [&](int n, uint32_t& bytes) -> const uint8_t* {
+    auto issue = [&](int n, int stg) {
       const int row = row0 + n / loads_per_row;
       const bool is_v = (loads_per_row == 2) ? (n & 1) : (rbk == 0);
-      const HeadEntry& h = is_v ? hv : hk;
-      bytes = is_v ? rbv : rbk;
-      return a.cache + row_offset(h.cache_off, bytes, gr.seq, row, a.page_table, a.pages_per_seq, a.rows_per_seq);
+      const uint32_t bytes = is_v ? rbv : rbk;
+      const uint8_t* src =
+          a.cache + row_offset(is_v ? voff : koff, bytes, gr.seq, row, a.page_table, a.pages_per_seq, a.rows_per_seq);
+      const uint32_t bar = smem_addr(&bars[stg]);
+      mbar_arrive_expect_tx(bar, bytes);
+      bulk_g2s(smem_addr(ring + (size_t)stg * stage_bytes), src, bytes, bar);
     };
-    // prologue: fill the ring
     int issued = 0;
-    if (lane == 0) {
-      for (; issued < n_loads && issued < nstage; ++issued) {
-        const int stg = (next_wait_stage + issued) % nstage;
-        uint32_t bytes;
-        const uint8_t* src = load_src(issued, bytes);
-        const uint32_t bar = smem_addr(&bars[stg]);
-        mbar_arrive_expect_tx(bar, bytes);
-        bulk_g2s(smem_addr(ring + (size_t)stg * stage_bytes), src, bytes, bar);
-      }
-    }
+    if (lane == 0)
+      for (; issued < n_loads && issued < nstage; ++issued) issue(issued, (next_wait_stage + issued) % nstage);
     issued = __shfl_sync(0xffffffffu, issued, 0);
     outstanding = issued;
 
-    int consumed = 0;
+    // wait for the next stage; returns its buffer or nullptr on timeout
+    auto acquire = [&]() -> const uint8_t* {
+      const int stg = next_wait_stage;
+      const bool ok =
+          __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&bars[stg]), (phase_bits >> stg) & 1u, kWaitLimitNs));
+      if (!ok) return nullptr;
+      phase_bits ^= 1u << stg;
+      return ring + (size_t)stg * stage_bytes;
+    };
+    // release the stage just consumed and refill it with the next load of this item
+    auto release = [&]() {
+      __syncwarp();
+      const int stg = next_wait_stage;
+      --outstanding;
+      next_wait_stage = (next_wait_stage + 1) % nstage;
+      if (issued < n_loads) {
+        if (lane == 0) {
+          fence_proxy_async_smem();
+          issue(issued, stg);
+        }
+        ++issued;
+        ++outstanding;
+      }
+    };
+
     for (int row = row0; row < row1; ++row) {
       float s[8][NT][2];
       // ---- K row ----
       if (rbk) {
-        const int stg = next_wait_stage;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&bars[stg]), (phase_bits >> stg) & 1u, kWaitLimitNs));
-        if (!ok) {
+        const uint8_t* buf = acquire();
+        if (!buf) {
           failed = true;
           break;
         }
-        phase_bits ^= 1u << stg;
-        k_row_dispatch<G>(hk.b, ring + (size_t)stg * stage_bytes, hk.r, bfrag, qsum, qscale, s);
-        __syncwarp();
-        ++consumed;
-        --outstanding;
-        next_wait_stage = (next_wait_stage + 1) % nstage;
-        if (lane == 0 && issued < n_loads) {
-          fence_proxy_async_smem();
-          uint32_t bytes;
-          const uint8_t* src = load_src(issued, bytes);
-          const uint32_t bar = smem_addr(&bars[stg]);
-          mbar_arrive_expect_tx(bar, bytes);
-          bulk_g2s(smem_addr(ring + (size_t)stg * stage_bytes), src, bytes, bar);
-        }
-        if (issued < n_loads) {
-          ++issued;
-          ++outstanding;
-        }
+        k_row_dispatch<G>(kb, buf, kr, bfrag, qg, qscale, s);
+        release();
       } else {
 #pragma unroll
         for (int t = 0; t < 8; ++t)
@@ -400,81 +414,75 @@ __global__ void __launch_bounds__(kDecodeWarps * 32) decode_kernel(DecodeArgs a)
           for (int nt = 0; nt < NT; ++nt) s[t][nt][0] = s[t][nt][1] = 0.f;
       }
       // ---- online softmax (base 2) ----
-      const int tbase = row * kRowTokens + (lane >> 2);
-      float p[8][NT][2];
+      // p is rounded to fp16 once; the rounded value feeds the V-side MMA, the running sum l
+      // and the offset correction alike, so the weights stay exactly normalised
+      if ((row + 1) * kRowTokens > T) {  // only the last row of a sequence has masked tokens
+        const int tbase = row * kRowTokens + (lane >> 2);
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int t = 0; t < 8; ++t) {
+            if (tbase + 16 * t >= T) s[t][nt][0] = -INFINITY;
+            if (tbase + 16 * t + 8 >= T) s[t][nt][1] = -INFINITY;
+          }
+      }
+      uint32_t bv[8][NT][2];
+      bool rescale = false;
+      float alpha[NT];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
         float mx = -INFINITY;
 #pragma unroll
-        for (int t = 0; t < 8; ++t) {
-          if (tbase + 16 * t >= T) s[t][nt][0] = -INFINITY;
-          if (tbase + 16 * t + 8 >= T) s[t][nt][1] = -INFINITY;
-          mx = fmaxf(mx, fmaxf(s[t][nt][0], s[t][nt][1]));
-        }
+        for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][nt][0], s[t][nt][1]));
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
         mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
         const float mnew = fmaxf(st.m[nt], mx);
-        const float alpha = exp2f(st.m[nt] - mnew);
+        alpha[nt] = ex2_approx(st.m[nt] - mnew);
+        rescale |= (mnew != st.m[nt]);
         st.m[nt] = mnew;
-        st.l[nt] *= alpha;
-        st.c[nt] *= alpha;
-#pragma unroll
-        for (int mu = 0; mu < 8; ++mu) {
-          st.o[nt][mu][0] *= alpha;
-          st.o[nt][mu][1] *= alpha;
-          st.o[nt][mu][2] *= alpha;
-          st.o[nt][mu][3] *= alpha;
-        }
-        float ls = 0.f;
+        float ls = 0.f, cs = 0.f;
 #pragma unroll
         for (int t = 0; t < 8; ++t) {
-          p[t][nt][0] = exp2f(s[t][nt][0] - mnew);
-          p[t][nt][1] = exp2f(s[t][nt][1] - mnew);
-          ls += p[t][nt][0] + p[t][nt][1];
+          const __half2 ph = __floats2half2_rn(ex2_approx(s[t][nt][0] - mnew), ex2_approx(s[t][nt][1] - mnew));
+          const float2 pf = __half22float2(ph);
+          ls += pf.x + pf.y;
+          if (vsmall) cs += pf.x * (vb == 1 ? Window<1>::off(2 * t) : Window<2>::off(2 * t)) +
+                            pf.y * (vb == 1 ? Window<1>::off(2 * t + 1) : Window<2>::off(2 * t + 1));
+          const uint32_t pw = *reinterpret_cast<const uint32_t*>(&ph);
+          bv[t][nt][0] = movmatrix_t(pw & 0xffffu);
+          bv[t][nt][1] = movmatrix_t(pw >> 16);
         }
-        st.l[nt] += ls;
+        st.l[nt] = st.l[nt] * alpha[nt] + ls;
+        st.c[nt] = st.c[nt] * alpha[nt] + cs;
       }
       // ---- V row ----
       if (rbv) {
-        uint32_t bv[8][NT][2];
+        if (__any_sync(0xffffffffu, rescale)) {
 #pragma unroll
-        for (int t = 0; t < 8; ++t)
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            const float h0 = __half2float(__float2half_rn(p[t][nt][0]));
-            const float h1 = __half2float(__float2half_rn(p[t][nt][1]));
-            bv[t][nt][0] = movmatrix_t(pack_f16(h0, p[t][nt][0] - h0));
-            bv[t][nt][1] = movmatrix_t(pack_f16(h1, p[t][nt][1] - h1));
-          }
-        const int stg = next_wait_stage;
-        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&bars[stg]), (phase_bits >> stg) & 1u, kWaitLimitNs));
-        if (!ok) {
+          for (int nt = 0; nt < NT; ++nt)
+            for (int mu = 0; mu < nmu; ++mu) {
+              float4* o = osm + (nt * 8 + mu) * 32 + lane;
+              float4 v = *o;
+              v.x *= alpha[nt];
+              v.y *= alpha[nt];
+              v.z *= alpha[nt];
+              v.w *= alpha[nt];
+              *o = v;
+            }
+        }
+        const uint8_t* buf = acquire();
+        if (!buf) {
           failed = true;
           break;
         }
-        phase_bits ^= 1u << stg;
-        v_row_dispatch<G>(hv.b, ring + (size_t)stg * stage_bytes, hv.r, bv, p, st);
-        __syncwarp();
-        ++consumed;
-        --outstanding;
-        next_wait_stage = (next_wait_stage + 1) % nstage;
-        if (lane == 0 && issued < n_loads) {
-          fence_proxy_async_smem();
-          uint32_t bytes;
-          const uint8_t* src = load_src(issued, bytes);
-          const uint32_t bar = smem_addr(&bars[stg]);
-          mbar_arrive_expect_tx(bar, bytes);
-          bulk_g2s(smem_addr(ring + (size_t)stg * stage_bytes), src, bytes, bar);
-        }
-        if (issued < n_loads) {
-          ++issued;
-          ++outstanding;
-        }
+        v_row_dispatch<G>(vb, buf, vr, bv, osm);
+        release();
       }
     }
     if (failed) break;
     // ---- write the partial of this item ----
+    __syncwarp();
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
       float l = st.l[nt], c = st.c[nt];
@@ -484,20 +492,21 @@ __global__ void __launch_bounds__(kDecodeWarps * 32) decode_kernel(DecodeArgs a)
       c += __shfl_xor_sync(0xffffffffu, c, 4);
       c += __shfl_xor_sync(0xffffffffu, c, 8);
       c += __shfl_xor_sync(0xffffffffu, c, 16);
+      if (!vsmall && vr > 0) c = (float)(1 << vb) * l;
       const int g = 4 * nt + (lane & 3);
       float* pg = part + g * gstride;
       if ((lane >> 2) == 0) {
         pg[0] = st.m[nt];
         pg[1] = l;
       }
-      const int rv = hv.r;
-#pragma unroll
-      for (int mu = 0; mu < 8; ++mu) {
+      for (int mu = 0; mu < nmu; ++mu) {
+        const float4 v = osm[(nt * 8 + mu) * 32 + lane];
         const int ch0 = 16 * mu + (lane >> 2), ch1 = ch0 + 8;
-        if (ch0 < rv) pg[4 + ch0] = (st.o[nt][mu][0] + st.o[nt][mu][1]) - c;
-        if (ch1 < rv) pg[4 + ch1] = (st.o[nt][mu][2] + st.o[nt][mu][3]) - c;
+        if (ch0 < vr) pg[4 + ch0] = (v.x + v.y) - c;
+        if (ch1 < vr) pg[4 + ch1] = (v.z + v.w) - c;
       }
     }
+    __syncwarp();
   }
   if (failed) {
     if (lane == 0) atomicOr(&g_status, 1u);

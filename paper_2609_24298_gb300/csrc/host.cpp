@@ -698,9 +698,27 @@ cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int*
     if (!d->pages_per_seq && rows > d->rows_per_seq) return COBRA_EINVAL;
     if (d->pages_per_seq && rows > 2LL * d->pages_per_seq) return COBRA_EINVAL;
   }
+  // groups ordered by (b_K, b_V, r_K, r_V, seq, layer, kv) so that the warps working on
+  // neighbouring chunks at the same time run the same code variant
+  struct Key {
+    int bk, bv, rk, rv, s, l, h;
+  };
+  std::vector<Key> keys;
   for (int s = 0; s < d->n_seqs; ++s)
     for (int l = 0; l < d->n_layers; ++l)
       for (int h = 0; h < d->n_kv_heads; ++h) {
+        const int hk = d->k_head0 + l * d->layer_stride + h, hv = d->v_head0 + l * d->layer_stride + h;
+        keys.push_back({head_r[hk] ? head_b[hk] : 0, head_r[hv] ? head_b[hv] : 0, head_r[hk], head_r[hv], s, l, h});
+      }
+  std::stable_sort(keys.begin(), keys.end(), [](const Key& x, const Key& y) {
+    if (x.bk != y.bk) return x.bk < y.bk;
+    if (x.bv != y.bv) return x.bv < y.bv;
+    if (x.rk != y.rk) return x.rk < y.rk;
+    return x.rv < y.rv;
+  });
+  for (const Key& key : keys) {
+      {
+        const int s = key.s, l = key.l, h = key.h;
         const int hk = d->k_head0 + l * d->layer_stride + h, hv = d->v_head0 + l * d->layer_stride + h;
         const int rk = head_r[hk], bk = head_r[hk] ? head_b[hk] : 0, rv = head_r[hv], bv = head_r[hv] ? head_b[hv] : 0;
         if (rk < 0 || rk > 128 || (rk & 1) || rv < 0 || rv > 128 || (rv & 1) || bk < 0 || bk > 8 || bv < 0 || bv > 8)
@@ -721,6 +739,7 @@ cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int*
         }
         p.groups.push_back(g);
       }
+  }
   return COBRA_OK;
 }
 

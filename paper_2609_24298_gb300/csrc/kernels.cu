@@ -130,7 +130,7 @@ cobra_status launch_decode(const DecodeArgs& a, int n_groups, int n_items, int s
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kScan) {
-    const size_t smem = (size_t)kDecodeWarps * a.nstage * (a.stage_bytes + 8);
+    const size_t smem = (size_t)kDecodeWarps * ((size_t)a.ring_bytes + (size_t)(G / 4) * 8 * 32 * 16 + kMaxStages * 8);
     static size_t attr_set = 0;
     if (smem > attr_set) {
       if (cudaFuncSetAttribute(decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
@@ -183,8 +183,8 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   a.rows_per_seq = d->rows_per_seq;
   a.pages_per_seq = d->pages_per_seq;
   const int rowb = info->max_row_bytes > 0 ? info->max_row_bytes : 16;
-  a.stage_bytes = (int)align_up((size_t)rowb, 128);
-  a.nstage = std::max(2, std::min(8, 24576 / a.stage_bytes));
+  // 8 KB of row staging per warp, or two of the largest rows if those are bigger
+  a.ring_bytes = (int)std::max<size_t>(8192, 2 * align_up((size_t)rowb, 128));
   cudaStream_t s = (cudaStream_t)stream;
   if (d->group == 4) return launch_decode<4>(a, info->n_groups, info->n_items, stages, s);
   return launch_decode<8>(a, info->n_groups, info->n_items, stages, s);
