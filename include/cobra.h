@@ -252,6 +252,32 @@ cobra_status cobra_decode_scan(const void* params, const cobra_decode_desc* desc
 cobra_status cobra_decode_combine(const void* params, const cobra_decode_desc* desc, const cobra_decode_info* info,
                                   const int* seq_lens, float* out, void* workspace, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------------------
+ * Decode attention without any device allocation.  (The paper has no counterpart; this is an
+ * interface convenience.)
+ *
+ * For callers that cannot allocate device memory - code running where cudaMalloc is not
+ * allowed or not wanted, such as an allocator's own callbacks, a process whose memory pool is
+ * fixed at start-up, or a plugin that must not touch the device heap - and so cannot provide
+ * the workspace cobra_decode_attn needs.  This call computes the same outputs, keeping its
+ * workspace in a fixed array of COBRA_STATIC_SCRATCH_BYTES bytes built into the library (it
+ * occupies that much memory on every GPU that loads the library, until the process exits).
+ *   - No plan or workspace argument: each call plans one token chunk per (seq, layer, kv
+ *     head) over the cache's capacity (rows_per_seq, or 2 * pages_per_seq rows when paged)
+ *     and writes that plan into the array itself, so nothing has to be zeroed beforehand.
+ *   - Returns COBRA_ESPACE when seqs x layers x kv heads chunks do not fit the array
+ *     (about 6.4 KB per chunk for group 4, 8.5 KB for group 8).
+ *   - The first call on each device looks up the array's address on that device (with the
+ *     device current); make that first call before any stream capture.
+ *   - All calls on a device share the one array and it keeps the last call's contents: calls
+ *     that can overlap on the GPU (different streams, no ordering between them) race and must
+ *     not be issued.
+ *   - Calls no cudaMalloc / cudaFree or any other allocating routine. */
+#define COBRA_STATIC_SCRATCH_BYTES (8u << 20)
+cobra_status cobra_decode_attn_static(const void* params, const cobra_decode_desc* desc, const void* q,
+                                      const uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
+                                      void* stream);
+
 /* Synchronise `stream`, then return and clear the device status word: COBRA_ETIMEOUT if a
  * bounded device wait expired since the last check, COBRA_EINVAL if a kernel skipped work
  * whose size did not fit its launch, COBRA_ECUDA on a CUDA error, else OK. */

@@ -80,6 +80,8 @@ SIGNATURES = {
                                   c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "cobra_decode_combine": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo), c_void_p,
                                      c_void_p, c_void_p, c_size_t, c_void_p]),
+    "cobra_decode_attn_static": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), c_void_p, c_void_p, c_void_p, c_void_p,
+                                         c_void_p, c_void_p]),
     "cobra_check": (c_int, [c_void_p]),
 }
 
@@ -306,6 +308,14 @@ def cobra_decode_combine(params, desc, info, seq_lens, out, workspace, ws_bytes:
     st = lib().cobra_decode_combine(_ptr(params), ctypes.byref(desc), ctypes.byref(info), _ptr(seq_lens), _ptr(out),
                                     _ptr(workspace), int(ws_bytes), _stream(stream))
     _chk("cobra_decode_combine", st)
+
+
+def cobra_decode_attn_static(params, desc: DecodeDesc, q, cache, seq_lens, page_table, out, stream=None):
+    """Decode attention for callers that cannot allocate device memory: the workspace is a
+    fixed array inside the library (see include/cobra.h)."""
+    st = lib().cobra_decode_attn_static(_ptr(params), ctypes.byref(desc), _ptr(q), _ptr(cache), _ptr(seq_lens),
+                                        _ptr(page_table), _ptr(out), _stream(stream))
+    _chk("cobra_decode_attn_static", st)
 
 
 def cobra_check(stream=None) -> int:

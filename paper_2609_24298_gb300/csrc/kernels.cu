@@ -3,6 +3,8 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
+#include <cstring>
 
 #include "../../include/cobra.h"
 #include "common.cuh"
@@ -217,6 +219,143 @@ extern "C" cobra_status cobra_decode_combine(const void* params, const cobra_dec
                                              void* workspace, size_t ws_bytes, void* stream) {
   return decode_common(params, d, info, nullptr, nullptr, seq_lens, nullptr, out, workspace, ws_bytes, stream,
                        kCombine);
+}
+
+// ---------------------------------------------------------------------------------------
+// Decode attention with library-owned scratch (no device allocation by anyone).
+//
+// Some callers cannot allocate device memory: code that runs where cudaMalloc is not allowed
+// or not wanted (inside an allocator's own callbacks, in a process whose memory pool is
+// fixed at start-up, or in a plugin that may not touch the device heap).  For them this entry
+// point keeps the decode workspace in one fixed array compiled into the library instead of
+// a caller buffer.  The array is kStaticScratchBytes long, lives on every GPU that loads the
+// library until the process exits, and is shared by every call on that GPU.
+// ---------------------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kStaticScratchBytes = COBRA_STATIC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::atomic<unsigned char*> g_scratch_ptr[kMaxDevices];
+
+// The host-side address of g_static_scratch on the current device, looked up once per device.
+cobra_status static_scratch(unsigned char** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return COBRA_ECUDA;
+  unsigned char* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
+  if (!p) {
+    void* addr = nullptr;
+    if (cudaGetSymbolAddress(&addr, g_static_scratch) != cudaSuccess || !addr) return COBRA_ECUDA;
+    p = static_cast<unsigned char*>(addr);
+    g_scratch_ptr[dev].store(p, std::memory_order_release);
+  }
+  *out = p;
+  return COBRA_OK;
+}
+
+// Workspace layout for a one-chunk-per-group plan with room for any head (r_V <= 128).
+struct StaticPlanSizes {
+  size_t groups_off, items_off, qt_off, part_off, total;
+  int g_stride, part_stride;
+};
+StaticPlanSizes static_plan_sizes(int n_groups, int group) {
+  StaticPlanSizes z{};
+  z.g_stride = 4 + kD;
+  z.part_stride = z.g_stride * group;
+  size_t off = align_up(sizeof(WsHeader), 256);
+  z.groups_off = off;
+  off = align_up(off + sizeof(WsGroup) * (size_t)n_groups, 256);
+  z.items_off = off;
+  off = align_up(off + sizeof(WsItem) * (size_t)n_groups, 256);
+  z.qt_off = off;
+  off = align_up(off + (size_t)kQtStride * n_groups, 256);
+  z.part_off = off;
+  off = align_up(off + sizeof(float) * (size_t)z.part_stride * n_groups, 256);
+  z.total = off;
+  return z;
+}
+
+// Writes the plan (header, groups, items) into the scratch: every (seq, layer, kv head) is one
+// chunk covering the sequence's whole capacity; the scan clips it to seq_lens.  Every field the
+// kernels read is rewritten on each call, so nothing has to start at zero.
+__global__ void static_plan_kernel(unsigned char* ws, const unsigned char* block, cobra_decode_desc d,
+                                   StaticPlanSizes z, int n_groups, int cap_rows) {
+  WsGroup* groups = reinterpret_cast<WsGroup*>(ws + z.groups_off);
+  WsItem* items = reinterpret_cast<WsItem*>(ws + z.items_off);
+  const HeadEntry* heads = head_table(block);
+  for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < n_groups; g += gridDim.x * blockDim.x) {
+    const int h = g % d.n_kv_heads, l = (g / d.n_kv_heads) % d.n_layers, s = g / (d.n_kv_heads * d.n_layers);
+    const int hk = d.k_head0 + l * d.layer_stride + h, hv = d.v_head0 + l * d.layer_stride + h;
+    groups[g] = WsGroup{s, l, h, g, 1, hk, hv, 0};
+    items[g] = WsItem{g, 0, cap_rows, 0};
+    (void)heads;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    WsHeader hd;
+    memset(&hd, 0, sizeof(hd));
+    hd.magic = kWsMagic;
+    hd.version = COBRA_VERSION;
+    hd.n_groups = n_groups;
+    hd.n_items = n_groups;
+    hd.group = d.group;
+    hd.n_layers = d.n_layers;
+    hd.n_kv = d.n_kv_heads;
+    hd.n_seqs = d.n_seqs;
+    hd.groups_off = z.groups_off;
+    hd.items_off = z.items_off;
+    hd.qt_off = z.qt_off;
+    hd.part_off = z.part_off;
+    hd.part_stride = z.part_stride;
+    hd.g_stride = z.g_stride;
+    hd.qt_stride = kQtStride;
+    hd.max_rv = kD;
+    hd.max_row_bytes = 16 * kD * 8;
+    *reinterpret_cast<WsHeader*>(ws) = hd;
+  }
+}
+
+}  // namespace
+
+extern "C" cobra_status cobra_decode_attn_static(const void* params, const cobra_decode_desc* d, const void* q,
+                                                 const uint8_t* cache, const int* seq_lens, const int* page_table,
+                                                 float* out, void* stream) {
+  if (!d || !params || !q || !cache || !seq_lens || !out) return COBRA_EINVAL;
+  if (d->n_layers < 1 || d->n_kv_heads < 1 || d->n_seqs < 1 || (d->group != 4 && d->group != 8) ||
+      d->layer_stride < d->n_kv_heads || d->k_head0 < 0 || d->v_head0 < 0)
+    return COBRA_EINVAL;
+  if (page_table ? d->pages_per_seq < 1 : d->rows_per_seq < 1) return COBRA_EINVAL;
+  if (!aligned(params, 256) || !aligned(cache, 256) || !aligned(out, 4) || !aligned(q, 2)) return COBRA_EALIGN;
+  const long long n_groups = (long long)d->n_seqs * d->n_layers * d->n_kv_heads;
+  if (n_groups > (1LL << 24)) return COBRA_ESPACE;
+  const StaticPlanSizes z = static_plan_sizes((int)n_groups, d->group);
+  if (z.total > kStaticScratchBytes) return COBRA_ESPACE;  // does not fit the fixed scratch
+  const int cap_rows = page_table ? 2 * d->pages_per_seq : d->rows_per_seq;
+  if (cap_rows > 65535) return COBRA_EINVAL;
+  unsigned char* ws = nullptr;
+  cobra_status st = static_scratch(&ws);
+  if (st != COBRA_OK) return st;
+  cudaStream_t s = (cudaStream_t)stream;
+  static_plan_kernel<<<(unsigned)std::min<long long>((n_groups + 255) / 256, 1024), 256, 0, s>>>(
+      ws, static_cast<const unsigned char*>(params), *d, z, (int)n_groups, cap_rows);
+  if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
+  DecodeArgs a{};
+  a.block = static_cast<const unsigned char*>(params);
+  a.cache = cache;
+  a.seq_lens = seq_lens;
+  a.page_table = page_table;
+  a.q = static_cast<const __nv_bfloat16*>(q);
+  a.out = out;
+  a.ws = ws;
+  a.q_sl = d->q_stride_layer;
+  a.q_ss = d->q_stride_seq;
+  a.o_sl = d->o_stride_layer;
+  a.o_ss = d->o_stride_seq;
+  a.rows_per_seq = d->rows_per_seq;
+  a.pages_per_seq = d->pages_per_seq;
+  a.ring_bytes = 2 * 16 * kD * 8;  // two rows of the largest head (r = 128, b = 8)
+  if (d->group == 4) return launch_decode<4>(a, (int)n_groups, (int)n_groups, kQproj | kScan | kCombine, s);
+  return launch_decode<8>(a, (int)n_groups, (int)n_groups, kQproj | kScan | kCombine, s);
 }
 
 extern "C" cobra_status cobra_check(void* stream) {
