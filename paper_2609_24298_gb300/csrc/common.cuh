@@ -101,21 +101,21 @@ __device__ __forceinline__ uint32_t pack_f16(float lo_col, float hi_col) {
 // ---------------------------------------------------------------------------------------
 // Unpacking one piece (b little-endian words, 32 codes) into 16 f16x2 registers.
 //
-// Register rho holds code (rho, 0) in its low half and code (rho, 1) in its high half, as
-// the f16 value off(rho) + code: the code is masked into mantissa bits [k, k+b) of a half
-// whose exponent field makes the value 2^(10-k) + code (k + b <= 10), so one AND/OR (plus
-// at most a shift) yields two codes.  off(rho) = 2^(10-k) is removed after the MMA.
+// Register rho holds code (rho, 0) in its low half and code (rho, 1) in its high half.  The
+// code is masked into mantissa bits [k, k+b) of an f16 whose other bits are those of 1.0
+// (kOneH2), so each half reads 1 + code * 2^(k-10): one AND/OR with an immediate mask and the
+// shared kOneH2 register (plus at most a shift) yields two codes.  The window k depends on
+// rho only; the unit offset and the per-window scale 2^(k-10) are removed after the MMA.
 // ---------------------------------------------------------------------------------------
-__host__ __device__ constexpr uint32_t magic2(int k) {
-  return ((uint32_t)(25 - k) << 10) | ((uint32_t)(25 - k) << 26);
-}
+constexpr uint32_t kOneH2 = 0x3C003C00u;  // f16 1.0 in both halves
+
 __host__ __device__ constexpr uint32_t pair_mask(int nbits, int k) {
   return (((1u << nbits) - 1u) << k) * 0x00010001u;
 }
 
 template <int B>
 struct Window {
-  // mantissa position used for register rho, and the matching offset 2^(10-k)
+  // mantissa position used for register rho
   __host__ __device__ static constexpr int k(int rho) {
     if (B == 1) return (rho >= 5 && rho <= 9) ? rho : (rho >= 10 && rho <= 14) ? rho - 5 : (rho <= 4) ? rho + 5 : 9;
     if (B == 2) {
@@ -124,7 +124,10 @@ struct Window {
     }
     return 10 - B;
   }
-  __host__ __device__ static constexpr float off(int rho) { return (float)(1 << (10 - k(rho))); }
+  // smallest window of this bit width (the reference the per-window scales are taken against)
+  __host__ __device__ static constexpr int kmin() { return B == 1 ? 5 : B == 2 ? 4 : 10 - B; }
+  // 2^(10-k): turns (value - 1) back into the code
+  __host__ __device__ static constexpr float inv_scale(int rho) { return (float)(1 << (10 - k(rho))); }
 };
 
 template <int B>
@@ -149,37 +152,37 @@ __host__ __device__ __forceinline__ void load_piece(const uint8_t* p, uint32_t (
 }
 
 // One register: codes (rho, 0) and (rho, 1) of the piece held in w.  rho is a compile-time
-// constant wherever this is called from an unrolled loop.
+// constant wherever this is called from an unrolled loop; `one` is kOneH2 held in a register.
 template <int B>
-__host__ __device__ __forceinline__ uint32_t unpack_reg(const uint32_t (&w)[B], int rho) {
+__host__ __device__ __forceinline__ uint32_t unpack_reg(const uint32_t (&w)[B], int rho, uint32_t one) {
   if constexpr (B == 1) {
     const int k = Window<1>::k(rho);
     const uint32_t x = w[0];
     const uint32_t t = (rho >= 5 && rho <= 9) ? x : (rho >= 10 && rho <= 14) ? (x >> 5) : (rho <= 4) ? (x << 5) : (x >> 6);
-    return (t & pair_mask(1, k)) | magic2(k);
+    return (t & pair_mask(1, k)) | one;
   } else if constexpr (B == 2) {
     const int l = rho & 7, k = Window<2>::k(rho);
     const uint32_t x = w[rho >> 3];
     const uint32_t t = (l >= 2 && l <= 4) ? x : (l >= 5) ? (x >> 6) : (x << 4);
-    return (t & pair_mask(2, k)) | magic2(k);
+    return (t & pair_mask(2, k)) | one;
   } else {
     constexpr int k = 10 - B;
     const int x = rho * B, wi = x >> 4, off = x & 15;
     if (off + B <= 16) {
       const uint32_t t = (off >= k) ? (w[wi] >> (off - k)) : (w[wi] << (k - off));
-      return (t & pair_mask(B, k)) | magic2(k);
+      return (t & pair_mask(B, k)) | one;
     }
     const int nlo = 16 - off;
     const uint32_t lo = w[wi] >> (off - k);
     const uint32_t hi = w[(wi + 1) < B ? wi + 1 : wi] << (k + nlo);
-    return (lo & pair_mask(nlo, k)) | (hi & pair_mask(B - nlo, k + nlo)) | magic2(k);
+    return (lo & pair_mask(nlo, k)) | (hi & pair_mask(B - nlo, k + nlo)) | one;
   }
 }
 
 template <int B>
 __host__ __device__ __forceinline__ void unpack_piece(const uint32_t (&w)[B], uint32_t (&o)[16]) {
 #pragma unroll
-  for (int rho = 0; rho < 16; ++rho) o[rho] = unpack_reg<B>(w, rho);
+  for (int rho = 0; rho < 16; ++rho) o[rho] = unpack_reg<B>(w, rho, kOneH2);
 }
 
 // Words of the piece at p, or zeros when the strip does not exist.

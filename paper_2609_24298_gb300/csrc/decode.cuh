@@ -34,6 +34,7 @@ struct DecodeArgs {
   long long q_sl, q_ss, o_sl, o_ss;
   int rows_per_seq, pages_per_seq;
   int ring_bytes;  // per-warp staging ring (>= 2 of the largest code rows, multiple of 128)
+  uint32_t one;    // kOneH2, passed at run time so that it stays in a register
 };
 
 // ---------------------------------------------------------------------------------------
@@ -151,7 +152,8 @@ struct WarpState {
 // (token t0 = 16 tau + lane/4 in [..][..][0], t1 = t0 + 8 in [..][..][1]), log2 units.
 template <int G, int B>
 __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const uint2* bfrag,
-                                             const float (&qg)[G / 4], float qscale, float (&s)[8][G / 4][2]) {
+                                             const float (&qsum)[G / 4], float qscale, uint32_t one,
+                                             float (&s)[8][G / 4][2]) {
   constexpr int NT = G / 4;
   const int lane = threadIdx.x & 31;
   float acc[8][NT][4];
@@ -175,24 +177,26 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
     for (int nt = 0; nt < NT; ++nt) bf[nt] = bfrag[(kap * 2 + nt) * 32 + lane];
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
-      const uint32_t a0 = unpack_reg<B>(wa, 2 * t), a1 = unpack_reg<B>(wa, 2 * t + 1);
-      const uint32_t a2 = unpack_reg<B>(wb, 2 * t), a3 = unpack_reg<B>(wb, 2 * t + 1);
+      const uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wa, 2 * t + 1, one);
+      const uint32_t a2 = unpack_reg<B>(wb, 2 * t, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) mma_f16(acc[t][nt], a0, a1, a2, a3, bf[nt].x, bf[nt].y);
     }
   }
-  // b >= 3 uses one window for every register, so the offset adds the same constant to every
-  // token's score and softmax ignores it; b = 1, 2 mix windows and need the per-token term
+  // acc = Qsum + 2^(k-10) * sum_i q~_i code_i, Qsum = sum of the q~ fed to the MMA.  b >= 3
+  // uses one window for every register, so Qsum shifts every token's score alike and softmax
+  // ignores it; b = 1, 2 mix windows, so Qsum is removed before the per-token rescale.
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
+      const float sc0 = qscale * Window<B>::inv_scale(2 * t), sc1 = qscale * Window<B>::inv_scale(2 * t + 1);
       if constexpr (B <= 2) {
-        s[t][nt][0] = fmaf(acc[t][nt][0] + acc[t][nt][1], qscale, -Window<B>::off(2 * t) * qg[nt]);
-        s[t][nt][1] = fmaf(acc[t][nt][2] + acc[t][nt][3], qscale, -Window<B>::off(2 * t + 1) * qg[nt]);
+        s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1] - qsum[nt]) * sc0;
+        s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3] - qsum[nt]) * sc1;
       } else {
-        s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1]) * qscale;
-        s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3]) * qscale;
+        s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1]) * sc0;
+        s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3]) * sc1;
       }
     }
   }
@@ -201,7 +205,7 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
 // V side: add one code row's rank-space contribution into the shared-memory accumulators.
 template <int G, int B>
 __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, const uint32_t (&bv)[8][G / 4][2],
-                                                 float4* osm) {
+                                                 uint32_t one, float4* osm) {
   constexpr int NT = G / 4;
   const int lane = threadIdx.x & 31;
   const int P = rv >> 1;
@@ -222,8 +226,8 @@ __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, c
       for (int u = 0; u < 2; ++u) d[nt][u][0] = d[nt][u][1] = d[nt][u][2] = d[nt][u][3] = 0.f;
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
-      const uint32_t a0 = unpack_reg<B>(wa, 2 * t), a1 = unpack_reg<B>(wb, 2 * t);
-      const uint32_t a2 = unpack_reg<B>(wa, 2 * t + 1), a3 = unpack_reg<B>(wb, 2 * t + 1);
+      const uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wb, 2 * t, one);
+      const uint32_t a2 = unpack_reg<B>(wa, 2 * t + 1, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) mma_f16(d[nt][t & 1], a0, a1, a2, a3, bv[t][nt][0], bv[t][nt][1]);
     }
@@ -242,37 +246,94 @@ __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, c
 
 template <int G>
 __device__ __forceinline__ void k_row_dispatch(int b, const uint8_t* stage, int rk, const uint2* bfrag,
-                                               const float (&qg)[G / 4], float qscale, float (&s)[8][G / 4][2]) {
+                                               const float (&qsum)[G / 4], float qscale, uint32_t one,
+                                               float (&s)[8][G / 4][2]) {
   switch (b) {
-    case 1: k_row_scores<G, 1>(stage, rk, bfrag, qg, qscale, s); break;
-    case 2: k_row_scores<G, 2>(stage, rk, bfrag, qg, qscale, s); break;
-    case 3: k_row_scores<G, 3>(stage, rk, bfrag, qg, qscale, s); break;
-    case 4: k_row_scores<G, 4>(stage, rk, bfrag, qg, qscale, s); break;
-    case 5: k_row_scores<G, 5>(stage, rk, bfrag, qg, qscale, s); break;
-    case 6: k_row_scores<G, 6>(stage, rk, bfrag, qg, qscale, s); break;
-    case 7: k_row_scores<G, 7>(stage, rk, bfrag, qg, qscale, s); break;
-    default: k_row_scores<G, 8>(stage, rk, bfrag, qg, qscale, s); break;
+    case 1: k_row_scores<G, 1>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    case 2: k_row_scores<G, 2>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    case 3: k_row_scores<G, 3>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    case 4: k_row_scores<G, 4>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    case 5: k_row_scores<G, 5>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    case 6: k_row_scores<G, 6>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    case 7: k_row_scores<G, 7>(stage, rk, bfrag, qsum, qscale, one, s); break;
+    default: k_row_scores<G, 8>(stage, rk, bfrag, qsum, qscale, one, s); break;
   }
 }
 
 template <int G>
 __device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int rv, const uint32_t (&bv)[8][G / 4][2],
-                                               float4* osm) {
+                                               uint32_t one, float4* osm) {
   switch (b) {
-    case 1: v_row_accumulate<G, 1>(stage, rv, bv, osm); break;
-    case 2: v_row_accumulate<G, 2>(stage, rv, bv, osm); break;
-    case 3: v_row_accumulate<G, 3>(stage, rv, bv, osm); break;
-    case 4: v_row_accumulate<G, 4>(stage, rv, bv, osm); break;
-    case 5: v_row_accumulate<G, 5>(stage, rv, bv, osm); break;
-    case 6: v_row_accumulate<G, 6>(stage, rv, bv, osm); break;
-    case 7: v_row_accumulate<G, 7>(stage, rv, bv, osm); break;
-    default: v_row_accumulate<G, 8>(stage, rv, bv, osm); break;
+    case 1: v_row_accumulate<G, 1>(stage, rv, bv, one, osm); break;
+    case 2: v_row_accumulate<G, 2>(stage, rv, bv, one, osm); break;
+    case 3: v_row_accumulate<G, 3>(stage, rv, bv, one, osm); break;
+    case 4: v_row_accumulate<G, 4>(stage, rv, bv, one, osm); break;
+    case 5: v_row_accumulate<G, 5>(stage, rv, bv, one, osm); break;
+    case 6: v_row_accumulate<G, 6>(stage, rv, bv, one, osm); break;
+    case 7: v_row_accumulate<G, 7>(stage, rv, bv, one, osm); break;
+    default: v_row_accumulate<G, 8>(stage, rv, bv, one, osm); break;
   }
 }
 
 template <int G>
 __device__ __forceinline__ size_t decode_osm_bytes() {
   return (size_t)(G / 4) * 8 * 32 * sizeof(float4);
+}
+
+// Online softmax of one row's scores (base 2) and the V-side MMA operands.  VC is the V bit
+// width's window class: 0 = one window for every register (b >= 3), 1 or 2 = the b = 1 / b = 2
+// windows.  V codes read 1 + code * 2^(k-10) with a per-register window k, so each token's
+// probability is fed to the MMA pre-scaled by 2^(kmin - k) (folded into the exponent): the
+// products then carry the single scale 2^(kmin-10), and the unit offsets add up to the plain
+// sum of the fed values, accumulated in c.  Every fed value is rounded to fp16 once and the
+// same rounded value enters l, c and the MMA, so the weights stay exactly normalised.
+template <int VC>
+struct VWin {
+  static constexpr int B = VC == 0 ? 3 : VC;
+  __device__ static constexpr float shift(int rho) {  // kmin - k (<= 0)
+    return VC == 0 ? 0.f : (float)(Window<B>::kmin() - Window<B>::k(rho));
+  }
+  __device__ static constexpr float unshift(int rho) {  // 2^(k - kmin)
+    return VC == 0 ? 1.f : (float)(1 << (Window<B>::k(rho) - Window<B>::kmin()));
+  }
+};
+
+template <int G, int VC>
+__device__ __forceinline__ void row_softmax(float (&s)[8][G / 4][2], WarpState<G>& st, float (&alpha)[G / 4],
+                                            bool& rescale, uint32_t (&bv)[8][G / 4][2]) {
+  constexpr int NT = G / 4;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    float mx = -INFINITY;
+#pragma unroll
+    for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][nt][0], s[t][nt][1]));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+    const float mnew = fmaxf(st.m[nt], mx);
+    alpha[nt] = ex2_approx(st.m[nt] - mnew);
+    rescale |= (mnew != st.m[nt]);
+    st.m[nt] = mnew;
+    float ls = 0.f, cs = 0.f;
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const float e0 = s[t][nt][0] - mnew + VWin<VC>::shift(2 * t);
+      const float e1 = s[t][nt][1] - mnew + VWin<VC>::shift(2 * t + 1);
+      const __half2 ph = __floats2half2_rn(ex2_approx(e0), ex2_approx(e1));
+      const float2 pf = __half22float2(ph);
+      if constexpr (VC == 0) {
+        ls += pf.x + pf.y;
+      } else {
+        ls += pf.x * VWin<VC>::unshift(2 * t) + pf.y * VWin<VC>::unshift(2 * t + 1);
+        cs += pf.x + pf.y;
+      }
+      const uint32_t pw = *reinterpret_cast<const uint32_t*>(&ph);
+      bv[t][nt][0] = movmatrix_t(pw & 0xffffu);
+      bv[t][nt][1] = movmatrix_t(pw >> 16);
+    }
+    st.l[nt] = st.l[nt] * alpha[nt] + ls;
+    st.c[nt] = st.c[nt] * alpha[nt] + cs;
+  }
 }
 
 template <int G>
@@ -300,9 +361,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
   const int gstride = wh->g_stride, pstride = wh->part_stride;
   uint32_t phase_bits = 0;  // parity of the next wait per barrier
   bool failed = false;
-  int outstanding = 0;      // loads issued but not yet waited for (stages are used in order)
-  int next_wait_stage = 0;
-  int nstage = 2, stage_bytes = ring_bytes / 2;
+  int outstanding = 0;      // loads issued but not yet waited for
+  int wait_stage = 0, nstage = 2;
 
   for (int item = blockIdx.x * kDecodeWarps + warp; item < n_items && !failed; item += gridDim.x * kDecodeWarps) {
     const WsItem it = items[item];
@@ -316,9 +376,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     const uint32_t rbk = kr > 0 ? 16u * kr * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
     // this item's stages: as many buffers of its largest row as the ring holds (every load of
     // the previous item has been consumed, so the ring is free)
-    stage_bytes = (int)((max(max(rbk, rbv), 16u) + 127u) & ~127u);
+    const int stage_bytes = (int)((max(max(rbk, rbv), 16u) + 127u) & ~127u);
     nstage = min(kMaxStages, ring_bytes / stage_bytes);
-    next_wait_stage = 0;
+    wait_stage = 0;
     if (nstage < 2) {
       // a row that does not fit the staging buffer is never copied; report and leave an
       // empty chunk (m = -inf, l = 0)
@@ -337,59 +397,67 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       st.c[nt] = 0.f;
     }
     const int nmu = ((vr >> 1) + 7) >> 3;
-    // V offsets: b >= 3 has one window, so the correction is 2^b * l (added at the end);
-    // b = 1, 2 need the per-token sum
-    const bool vsmall = vr > 0 && vb <= 2;
     for (int k = 0; k < NT * nmu; ++k) {
       const int nt = k / nmu, mu = k % nmu;
       osm[(nt * 8 + mu) * 32 + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    const int loads_per_row = (rbk ? 1 : 0) + (rbv ? 1 : 0);
-    const int n_loads = row1 > row0 ? (row1 - row0) * loads_per_row : 0;
+    // V window class (see row_softmax) and the factor 2^(10 - kmin) that turns the fed
+    // products back into codes
+    const int vc = (vr > 0 && vb <= 2) ? vb : 0;
+    const float vout = vr == 0 ? 0.f : (float)(1 << (vb == 1 ? 5 : vb == 2 ? 6 : vb));
+    const bool two = rbk && rbv;
+    const int n_loads = row1 > row0 ? (row1 - row0) * (two ? 2 : (rbk || rbv ? 1 : 0)) : 0;
     const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
     const float* qhdr = reinterpret_cast<const float*>(qt);
     const uint2* bfrag = reinterpret_cast<const uint2*>(qt + kQtHeaderBytes);
-    float qg[NT];
+    float qsum[NT];
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) qg[nt] = qhdr[4 * nt + (lane & 3)] * qhdr[8];
+    for (int nt = 0; nt < NT; ++nt) qsum[nt] = qhdr[4 * nt + (lane & 3)];
     const float qscale = qhdr[8];
+    const uint32_t one = a.one;
 
-    // load n of this item -> (row, side)
-    auto issue = [&](int n, int stg) {
-      const int row = row0 + n / loads_per_row;
-      const bool is_v = (loads_per_row == 2) ? (n & 1) : (rbk == 0);
-      const uint32_t bytes = is_v ? rbv : rbk;
-      const uint8_t* src =
-          a.cache + row_offset(is_v ? voff : koff, bytes, gr.seq, row, a.page_table, a.pages_per_seq, a.rows_per_seq);
-      const uint32_t bar = smem_addr(&bars[stg]);
+    // issue state (lane 0 only): next row / side / stage to load
+    int iss_row = row0, iss_stage = 0;
+    bool iss_v = !rbk;
+    const uint8_t* kbase = a.cache + koff;
+    const uint8_t* vbase = a.cache + voff;
+    auto issue_next = [&]() {
+      const uint32_t bytes = iss_v ? rbv : rbk;
+      const uint8_t* src = (iss_v ? vbase : kbase) +
+                           row_offset(0, bytes, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq);
+      const uint32_t bar = smem_addr(&bars[iss_stage]);
       mbar_arrive_expect_tx(bar, bytes);
-      bulk_g2s(smem_addr(ring + (size_t)stg * stage_bytes), src, bytes, bar);
+      bulk_g2s(smem_addr(ring + (size_t)iss_stage * stage_bytes), src, bytes, bar);
+      if (two && !iss_v) {
+        iss_v = true;
+      } else {
+        iss_v = !rbk;
+        ++iss_row;
+      }
+      if (++iss_stage == nstage) iss_stage = 0;
     };
-    int issued = 0;
+    int issued = min(n_loads, nstage);
     if (lane == 0)
-      for (; issued < n_loads && issued < nstage; ++issued) issue(issued, (next_wait_stage + issued) % nstage);
-    issued = __shfl_sync(0xffffffffu, issued, 0);
+      for (int k = 0; k < issued; ++k) issue_next();
     outstanding = issued;
 
     // wait for the next stage; returns its buffer or nullptr on timeout
     auto acquire = [&]() -> const uint8_t* {
-      const int stg = next_wait_stage;
-      const bool ok =
-          __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&bars[stg]), (phase_bits >> stg) & 1u, kWaitLimitNs));
+      const bool ok = __all_sync(
+          0xffffffffu, mbar_wait_bounded(smem_addr(&bars[wait_stage]), (phase_bits >> wait_stage) & 1u, kWaitLimitNs));
       if (!ok) return nullptr;
-      phase_bits ^= 1u << stg;
-      return ring + (size_t)stg * stage_bytes;
+      phase_bits ^= 1u << wait_stage;
+      return ring + (size_t)wait_stage * stage_bytes;
     };
     // release the stage just consumed and refill it with the next load of this item
     auto release = [&]() {
       __syncwarp();
-      const int stg = next_wait_stage;
       --outstanding;
-      next_wait_stage = (next_wait_stage + 1) % nstage;
+      if (++wait_stage == nstage) wait_stage = 0;
       if (issued < n_loads) {
         if (lane == 0) {
           fence_proxy_async_smem();
-          issue(issued, stg);
+          issue_next();
         }
         ++issued;
         ++outstanding;
@@ -405,7 +473,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
           failed = true;
           break;
         }
-        k_row_dispatch<G>(kb, buf, kr, bfrag, qg, qscale, s);
+        k_row_dispatch<G>(kb, buf, kr, bfrag, qsum, qscale, one, s);
         release();
       } else {
 #pragma unroll
@@ -413,9 +481,6 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) s[t][nt][0] = s[t][nt][1] = 0.f;
       }
-      // ---- online softmax (base 2) ----
-      // p is rounded to fp16 once; the rounded value feeds the V-side MMA, the running sum l
-      // and the offset correction alike, so the weights stay exactly normalised
       if ((row + 1) * kRowTokens > T) {  // only the last row of a sequence has masked tokens
         const int tbase = row * kRowTokens + (lane >> 2);
 #pragma unroll
@@ -429,33 +494,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       uint32_t bv[8][NT][2];
       bool rescale = false;
       float alpha[NT];
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        float mx = -INFINITY;
-#pragma unroll
-        for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][nt][0], s[t][nt][1]));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-        const float mnew = fmaxf(st.m[nt], mx);
-        alpha[nt] = ex2_approx(st.m[nt] - mnew);
-        rescale |= (mnew != st.m[nt]);
-        st.m[nt] = mnew;
-        float ls = 0.f, cs = 0.f;
-#pragma unroll
-        for (int t = 0; t < 8; ++t) {
-          const __half2 ph = __floats2half2_rn(ex2_approx(s[t][nt][0] - mnew), ex2_approx(s[t][nt][1] - mnew));
-          const float2 pf = __half22float2(ph);
-          ls += pf.x + pf.y;
-          if (vsmall) cs += pf.x * (vb == 1 ? Window<1>::off(2 * t) : Window<2>::off(2 * t)) +
-                            pf.y * (vb == 1 ? Window<1>::off(2 * t + 1) : Window<2>::off(2 * t + 1));
-          const uint32_t pw = *reinterpret_cast<const uint32_t*>(&ph);
-          bv[t][nt][0] = movmatrix_t(pw & 0xffffu);
-          bv[t][nt][1] = movmatrix_t(pw >> 16);
-        }
-        st.l[nt] = st.l[nt] * alpha[nt] + ls;
-        st.c[nt] = st.c[nt] * alpha[nt] + cs;
-      }
+      if (vc == 1)
+        row_softmax<G, 1>(s, st, alpha, rescale, bv);
+      else if (vc == 2)
+        row_softmax<G, 2>(s, st, alpha, rescale, bv);
+      else
+        row_softmax<G, 0>(s, st, alpha, rescale, bv);
       // ---- V row ----
       if (rbv) {
         if (__any_sync(0xffffffffu, rescale)) {
@@ -476,7 +520,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
           failed = true;
           break;
         }
-        v_row_dispatch<G>(vb, buf, vr, bv, osm);
+        v_row_dispatch<G>(vb, buf, vr, bv, one, osm);
         release();
       }
     }
@@ -492,7 +536,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       c += __shfl_xor_sync(0xffffffffu, c, 4);
       c += __shfl_xor_sync(0xffffffffu, c, 8);
       c += __shfl_xor_sync(0xffffffffu, c, 16);
-      if (!vsmall && vr > 0) c = (float)(1 << vb) * l;
+      if (vc == 0) c = l;
       const int g = 4 * nt + (lane & 3);
       float* pg = part + g * gstride;
       if ((lane >> 2) == 0) {
@@ -502,8 +546,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       for (int mu = 0; mu < nmu; ++mu) {
         const float4 v = osm[(nt * 8 + mu) * 32 + lane];
         const int ch0 = 16 * mu + (lane >> 2), ch1 = ch0 + 8;
-        if (ch0 < vr) pg[4 + ch0] = (v.x + v.y) - c;
-        if (ch1 < vr) pg[4 + ch1] = (v.z + v.w) - c;
+        if (ch0 < vr) pg[4 + ch0] = ((v.x + v.y) - c) * vout;
+        if (ch1 < vr) pg[4 + ch1] = ((v.z + v.w) - c) * vout;
       }
     }
     __syncwarp();
@@ -512,9 +556,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     if (lane == 0) atomicOr(&g_status, 1u);
     // drain the copies still in flight before the shared memory goes away
     for (int k = 0; k < outstanding; ++k) {
-      const int stg = (next_wait_stage + k) % nstage;
-      if (!mbar_wait_bounded(smem_addr(&bars[stg]), (phase_bits >> stg) & 1u, kWaitLimitNs)) break;
-      phase_bits ^= 1u << stg;
+      if (!mbar_wait_bounded(smem_addr(&bars[wait_stage]), (phase_bits >> wait_stage) & 1u, kWaitLimitNs)) break;
+      phase_bits ^= 1u << wait_stage;
+      if (++wait_stage == nstage) wait_stage = 0;
     }
   }
 }

@@ -184,6 +184,7 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   a.o_ss = d->o_stride_seq;
   a.rows_per_seq = d->rows_per_seq;
   a.pages_per_seq = d->pages_per_seq;
+  a.one = kOneH2;
   const int rowb = info->max_row_bytes > 0 ? info->max_row_bytes : 16;
   // 8 KB of row staging per warp, or two of the largest rows if those are bigger
   a.ring_bytes = (int)std::max<size_t>(8192, 2 * align_up((size_t)rowb, 128));
@@ -353,6 +354,7 @@ extern "C" cobra_status cobra_decode_attn_static(const void* params, const cobra
   a.o_ss = d->o_stride_seq;
   a.rows_per_seq = d->rows_per_seq;
   a.pages_per_seq = d->pages_per_seq;
+  a.one = kOneH2;
   a.ring_bytes = 2 * 16 * kD * 8;  // two rows of the largest head (r = 128, b = 8)
   if (d->group == 4) return launch_decode<4>(a, (int)n_groups, (int)n_groups, kQproj | kScan | kCombine, s);
   return launch_decode<8>(a, (int)n_groups, (int)n_groups, kQproj | kScan | kCombine, s);
