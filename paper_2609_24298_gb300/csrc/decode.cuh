@@ -7,12 +7,22 @@
 //                   Each warp streams its chunk's K and V code rows into a private shared-
 //                   memory ring with bulk async copies, unpacks codes in registers and runs
 //                   f16 mma.sync with fp32 accumulation:
-//                     scores  S[t][(g,hi|lo)] = sum_i code^K[t][i] q~[i][(g,hi|lo)]   (M = tokens)
-//                     values  O[i][(g,hi|lo)] += sum_t code^V[t][i] P[t][(g,hi|lo)]  (M = channels)
+//                     scores  S[t][col] = sum_i code^K[t][i] q~[i][col]   (M = tokens, K = channels)
+//                     values  O[i][g]  += sum_t code^V[t][i] P[t][g]      (M = channels, K = tokens)
 //                   with an online softmax in base 2 between them.  Writes per-chunk
 //                   partials (m, l, sum_t p_t c^V_t).
 //   combine_kernel  merges the chunks of each (seq, layer, kv-head), dequantises the rank-space
 //                   average and back-projects once: o = mu_V + W_V Delta_V (acc/l - 2^{b-1} + 1/2).
+//
+// Query heads per lane.  Lane l (j = l % 4) owns NG = G / 4 query heads:
+//   G = 4: head j.  Score columns are interleaved (head g hi, head g lo) in one n-tile, so the
+//          lane's columns 2j, 2j+1 are the hi and lo parts of head j; the V side's B operand
+//          holds (p_j, 0) in columns (2j, 2j+1).
+//   G = 8: heads 2j, 2j+1.  Scores use two n-tiles (q~ hi for heads 0..7 | q~ lo for heads
+//          0..7), so the lane's columns 2j, 2j+1 are its two heads in both; the V side's B
+//          operand holds (p_2j, p_2j+1).
+// Either way the probabilities of a 16-token tile sit in the MMA C-fragment layout and one
+// movmatrix per 8 tokens turns them into the V side's B fragment.
 #pragma once
 
 #include "common.cuh"
@@ -37,12 +47,23 @@ struct DecodeArgs {
   uint32_t one;    // kOneH2, passed at run time so that it stays in a register
 };
 
+template <int G>
+struct Heads {
+  static constexpr int NG = G / 4;  // query heads per lane
+  static constexpr int NTK = G / 4; // score n-tiles
+  // query head of score column n in n-tile nt, and whether that column holds the lo part
+  __host__ __device__ static constexpr int col_head(int nt, int n) { return G == 4 ? n >> 1 : n; }
+  __host__ __device__ static constexpr int col_lo(int nt, int n) { return G == 4 ? (n & 1) : nt; }
+  // the lane's u-th query head (j = lane % 4)
+  __device__ static int head(int j, int u) { return G == 4 ? j : 2 * j + u; }
+};
+
 // ---------------------------------------------------------------------------------------
 // a4: query projection
 // ---------------------------------------------------------------------------------------
 template <int G>
 __global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
-  constexpr int NT = G / 4;
+  constexpr int NTK = Heads<G>::NTK;
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup gr = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off)[blockIdx.x];
   const HeadEntry hk = head_table(a.block)[gr.k_head];
@@ -61,10 +82,10 @@ __global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
   const float scale = hk.delta * 0.088388347648318440f * 1.4426950408889634f;  // Delta/sqrt(128)*log2(e)
   float vals[G];
   float amax = 0.f;
+#pragma unroll
+  for (int g = 0; g < G; ++g) vals[g] = 0.f;
   if (tid < r) {
     const float* w = pool + hk.w_off + (size_t)tid * kD;
-#pragma unroll
-    for (int g = 0; g < G; ++g) vals[g] = 0.f;
     for (int dd = 0; dd < kD; dd += 4) {
       const float4 wv = *reinterpret_cast<const float4*>(w + dd);
 #pragma unroll
@@ -76,9 +97,6 @@ __global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
       vals[g] *= scale;
       amax = fmaxf(amax, fabsf(vals[g]));
     }
-  } else {
-#pragma unroll
-    for (int g = 0; g < G; ++g) vals[g] = 0.f;
   }
   // power-of-two scale so that max |q~| lands in [256, 512)
 #pragma unroll
@@ -109,13 +127,13 @@ __global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
     qhdr[tid] = s;
   }
   if (tid == 0) qhdr[8] = ldexpf(1.f, -e);
-  // B fragments: [kappa][nt][lane] uint2; element (k, n): channel 16 kappa + k, column n =
-  // 2 (g mod 4) + (hi|lo) of query head g = 4 nt + n / 2.
+  // B fragments [kappa][nt][lane] uint2: element (k, n) = hi or lo part of q~ of channel
+  // 16 kappa + k for the query head of column n (see Heads)
   uint2* frag = reinterpret_cast<uint2*>(qt + kQtHeaderBytes);
-  for (int idx = tid; idx < 8 * NT * 32; idx += 128) {
-    const int lane = idx & 31, nt = (idx >> 5) % NT, kap = idx / (32 * NT);
+  for (int idx = tid; idx < 8 * NTK * 32; idx += 128) {
+    const int lane = idx & 31, nt = (idx >> 5) % NTK, kap = idx / (32 * NTK);
     const int j = lane & 3, n = lane >> 2;
-    const int g = 4 * nt + (n >> 1), lo = n & 1;
+    const int g = Heads<G>::col_head(nt, n), lo = Heads<G>::col_lo(nt, n);
     float e4[4];
     const int ks[4] = {2 * j, 2 * j + 1, 2 * j + 8, 2 * j + 9};
 #pragma unroll
@@ -136,67 +154,88 @@ __global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
 // ---------------------------------------------------------------------------------------
 // a5 + a6: chunked rank-space scan
 //
-// Per warp: running max m, sum l and offset correction c per query head in registers; the
-// rank-space value accumulators O[nt][mu] (lane-owned float4 of the MMA C fragment) live in
-// the warp's shared memory and are rescaled only when the running max moves.  Loops over
-// k-tiles (K side) and channel tiles (V side) stay rolled to keep each (b_K, b_V) variant's
-// code small; only the 8 token tiles of a row are unrolled.
+// Per warp: running max m, sum l and offset correction c per owned query head in registers;
+// the rank-space value accumulators (the lane's C-fragment entries of O) live in the warp's
+// shared memory and are rescaled only when the running max moves.  Loops over k-tiles (K
+// side) and channel tiles (V side) stay rolled to keep each (b_K, b_V) variant's code small;
+// only the 8 token tiles of a row are unrolled.
 // ---------------------------------------------------------------------------------------
 template <int G>
 struct WarpState {
-  static constexpr int NT = G / 4;
-  float m[NT], l[NT], c[NT];
+  static constexpr int NG = G / 4;
+  float m[NG], l[NG], c[NG];
 };
 
-// K side: scores of one code row for the lane's query heads, s[8][NT][2]
+// accumulator floats per (channel tile, lane): the live C-fragment entries of the V MMA
+template <int G>
+struct OAcc {
+  static constexpr int N = G == 4 ? 2 : 4;  // G = 4: columns 2j only; G = 8: both columns
+};
+
+// K side: scores of one code row for the lane's query heads, s[8][NG][2]
 // (token t0 = 16 tau + lane/4 in [..][..][0], t1 = t0 + 8 in [..][..][1]), log2 units.
 template <int G, int B>
 __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const uint2* bfrag,
                                              const float (&qsum)[G / 4], float qscale, uint32_t one,
                                              float (&s)[8][G / 4][2]) {
-  constexpr int NT = G / 4;
+  constexpr int NTK = Heads<G>::NTK, NG = Heads<G>::NG;
   const int lane = threadIdx.x & 31;
-  float acc[8][NT][4];
+  float acc[8][NTK][4];
 #pragma unroll
   for (int t = 0; t < 8; ++t)
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) acc[t][nt][0] = acc[t][nt][1] = acc[t][nt][2] = acc[t][nt][3] = 0.f;
+    for (int nt = 0; nt < NTK; ++nt) acc[t][nt][0] = acc[t][nt][1] = acc[t][nt][2] = acc[t][nt][3] = 0.f;
   const int P = rk >> 1;
-  const int nk = (P + 7) >> 3;
-  const int pc = lane >> 2;
-#pragma unroll 1
-  for (int kap = 0; kap < nk; ++kap) {
+  const int nfull = P >> 3, nk = (P + 7) >> 3;
+  // lane's pieces: strips 8 kappa + (lane & 3) and + 4, piece lane >> 2
+  const uint8_t* pa = stage + (lane & 3) * 32 * B + (lane >> 2) * 4 * B;
+  const uint2* bq = bfrag + lane;
+  auto tile = [&](bool check, int kap) {
     // channels past r (a partial last k-tile) multiply q~ = 0, so their operand values only
     // need to be finite; the words are zeroed rather than read past the row
-    const int sA = 8 * kap + (lane & 3), sB = sA + 4;
     uint32_t wa[B], wb[B];
-    load_piece_or_zero<B>(stage + sA * 32 * B + pc * 4 * B, sA < P, wa);
-    load_piece_or_zero<B>(stage + sB * 32 * B + pc * 4 * B, sB < P, wb);
-    uint2 bf[NT];
+    if (check) {
+      const int sA = 8 * kap + (lane & 3);
+      load_piece_or_zero<B>(pa, sA < P, wa);
+      load_piece_or_zero<B>(pa + 4 * 32 * B, sA + 4 < P, wb);
+    } else {
+      load_piece<B>(pa, wa);
+      load_piece<B>(pa + 4 * 32 * B, wb);
+    }
+    uint2 bf[NTK];
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) bf[nt] = bfrag[(kap * 2 + nt) * 32 + lane];
+    for (int nt = 0; nt < NTK; ++nt) bf[nt] = bq[nt * 32];
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
       const uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wa, 2 * t + 1, one);
       const uint32_t a2 = unpack_reg<B>(wb, 2 * t, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) mma_f16(acc[t][nt], a0, a1, a2, a3, bf[nt].x, bf[nt].y);
+      for (int nt = 0; nt < NTK; ++nt) mma_f16(acc[t][nt], a0, a1, a2, a3, bf[nt].x, bf[nt].y);
     }
-  }
+    pa += 8 * 32 * B;
+    bq += 2 * 32;
+  };
+#pragma unroll 1
+  for (int kap = 0; kap < nfull; ++kap) tile(false, kap);
+  if (nk > nfull) tile(true, nfull);
   // acc = Qsum + 2^(k-10) * sum_i q~_i code_i, Qsum = sum of the q~ fed to the MMA.  b >= 3
   // uses one window for every register, so Qsum shifts every token's score alike and softmax
   // ignores it; b = 1, 2 mix windows, so Qsum is removed before the per-token rescale.
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
+  for (int t = 0; t < 8; ++t) {
+    const float sc0 = qscale * Window<B>::inv_scale(2 * t), sc1 = qscale * Window<B>::inv_scale(2 * t + 1);
 #pragma unroll
-    for (int t = 0; t < 8; ++t) {
-      const float sc0 = qscale * Window<B>::inv_scale(2 * t), sc1 = qscale * Window<B>::inv_scale(2 * t + 1);
+    for (int u = 0; u < NG; ++u) {
+      // hi + lo parts of the u-th head: G = 4 -> columns (2j, 2j+1) of n-tile 0;
+      // G = 8 -> column 2j + u of n-tiles 0 and 1
+      const float v0 = G == 4 ? acc[t][0][0] + acc[t][0][1] : acc[t][0][u] + acc[t][NTK - 1][u];
+      const float v1 = G == 4 ? acc[t][0][2] + acc[t][0][3] : acc[t][0][2 + u] + acc[t][NTK - 1][2 + u];
       if constexpr (B <= 2) {
-        s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1] - qsum[nt]) * sc0;
-        s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3] - qsum[nt]) * sc1;
+        s[t][u][0] = (v0 - qsum[u]) * sc0;
+        s[t][u][1] = (v1 - qsum[u]) * sc1;
       } else {
-        s[t][nt][0] = (acc[t][nt][0] + acc[t][nt][1]) * sc0;
-        s[t][nt][1] = (acc[t][nt][2] + acc[t][nt][3]) * sc1;
+        s[t][u][0] = v0 * sc0;
+        s[t][u][1] = v1 * sc1;
       }
     }
   }
@@ -204,44 +243,55 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
 
 // V side: add one code row's rank-space contribution into the shared-memory accumulators.
 template <int G, int B>
-__device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, const uint32_t (&bv)[8][G / 4][2],
-                                                 uint32_t one, float4* osm) {
-  constexpr int NT = G / 4;
+__device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, const uint32_t (&bv)[8][2],
+                                                 uint32_t one, float* osm) {
+  constexpr int NO = OAcc<G>::N;
   const int lane = threadIdx.x & 31;
   const int P = rv >> 1;
-  const int nmu = (P + 7) >> 3;
-  const int pc = lane & 7;
-#pragma unroll 1
-  for (int mu = 0; mu < nmu; ++mu) {
+  const int nfull = P >> 3, nmu = (P + 7) >> 3;
+  // lane's pieces: strips 8 mu + (lane >> 3) and + 4, piece lane & 7
+  const uint8_t* pa = stage + (lane >> 3) * 32 * B + (lane & 7) * 4 * B;
+  float* o = osm + lane * NO;
+  auto tile = [&](bool check, int mu) {
     // rows for channels past r are never written out, so their operand values only need to
     // be finite
-    const int sA = 8 * mu + (lane >> 3), sB = sA + 4;
     uint32_t wa[B], wb[B];
-    load_piece_or_zero<B>(stage + sA * 32 * B + pc * 4 * B, sA < P, wa);
-    load_piece_or_zero<B>(stage + sB * 32 * B + pc * 4 * B, sB < P, wb);
-    float d[NT][2][4];
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-      for (int u = 0; u < 2; ++u) d[nt][u][0] = d[nt][u][1] = d[nt][u][2] = d[nt][u][3] = 0.f;
+    if (check) {
+      const int sA = 8 * mu + (lane >> 3);
+      load_piece_or_zero<B>(pa, sA < P, wa);
+      load_piece_or_zero<B>(pa + 4 * 32 * B, sA + 4 < P, wb);
+    } else {
+      load_piece<B>(pa, wa);
+      load_piece<B>(pa + 4 * 32 * B, wb);
+    }
+    // fresh accumulators per row: the running sums in shared memory are dominated by the unit
+    // code offsets, so they are only ever updated with round-to-nearest fp32 adds
+    float d[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
       const uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wb, 2 * t, one);
       const uint32_t a2 = unpack_reg<B>(wa, 2 * t + 1, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) mma_f16(d[nt][t & 1], a0, a1, a2, a3, bv[t][nt][0], bv[t][nt][1]);
+      mma_f16(d[t & 1], a0, a1, a2, a3, bv[t][0], bv[t][1]);
     }
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      float4* o = osm + (nt * 8 + mu) * 32 + lane;
-      float4 v = *o;
-      v.x += d[nt][0][0] + d[nt][1][0];
-      v.y += d[nt][0][1] + d[nt][1][1];
-      v.z += d[nt][0][2] + d[nt][1][2];
-      v.w += d[nt][0][3] + d[nt][1][3];
-      *o = v;
+    if constexpr (NO == 2) {
+      float2 v = *reinterpret_cast<float2*>(o);
+      v.x += d[0][0] + d[1][0];
+      v.y += d[0][2] + d[1][2];
+      *reinterpret_cast<float2*>(o) = v;
+    } else {
+      float4 v = *reinterpret_cast<float4*>(o);
+      v.x += d[0][0] + d[1][0];
+      v.y += d[0][1] + d[1][1];
+      v.z += d[0][2] + d[1][2];
+      v.w += d[0][3] + d[1][3];
+      *reinterpret_cast<float4*>(o) = v;
     }
-  }
+    pa += 8 * 32 * B;
+    o += 32 * NO;
+  };
+#pragma unroll 1
+  for (int mu = 0; mu < nfull; ++mu) tile(false, mu);
+  if (nmu > nfull) tile(true, nfull);
 }
 
 template <int G>
@@ -261,8 +311,8 @@ __device__ __forceinline__ void k_row_dispatch(int b, const uint8_t* stage, int 
 }
 
 template <int G>
-__device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int rv, const uint32_t (&bv)[8][G / 4][2],
-                                               uint32_t one, float4* osm) {
+__device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int rv, const uint32_t (&bv)[8][2],
+                                               uint32_t one, float* osm) {
   switch (b) {
     case 1: v_row_accumulate<G, 1>(stage, rv, bv, one, osm); break;
     case 2: v_row_accumulate<G, 2>(stage, rv, bv, one, osm); break;
@@ -277,7 +327,7 @@ __device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int 
 
 template <int G>
 __device__ __forceinline__ size_t decode_osm_bytes() {
-  return (size_t)(G / 4) * 8 * 32 * sizeof(float4);
+  return (size_t)8 * 32 * OAcc<G>::N * sizeof(float);
 }
 
 // Online softmax of one row's scores (base 2) and the V-side MMA operands.  VC is the V bit
@@ -300,51 +350,60 @@ struct VWin {
 
 template <int G, int VC>
 __device__ __forceinline__ void row_softmax(float (&s)[8][G / 4][2], WarpState<G>& st, float (&alpha)[G / 4],
-                                            bool& rescale, uint32_t (&bv)[8][G / 4][2]) {
-  constexpr int NT = G / 4;
+                                            bool& rescale, uint32_t (&bv)[8][2]) {
+  constexpr int NG = G / 4;
+  float pf[8][NG][2];
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
+  for (int u = 0; u < NG; ++u) {
     float mx = -INFINITY;
 #pragma unroll
-    for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][nt][0], s[t][nt][1]));
+    for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][u][0], s[t][u][1]));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-    const float mnew = fmaxf(st.m[nt], mx);
-    alpha[nt] = ex2_approx(st.m[nt] - mnew);
-    rescale |= (mnew != st.m[nt]);
-    st.m[nt] = mnew;
+    const float mnew = fmaxf(st.m[u], mx);
+    alpha[u] = ex2_approx(st.m[u] - mnew);
+    rescale |= (mnew != st.m[u]);
+    st.m[u] = mnew;
     float ls = 0.f, cs = 0.f;
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
-      const float e0 = s[t][nt][0] - mnew + VWin<VC>::shift(2 * t);
-      const float e1 = s[t][nt][1] - mnew + VWin<VC>::shift(2 * t + 1);
-      const __half2 ph = __floats2half2_rn(ex2_approx(e0), ex2_approx(e1));
-      const float2 pf = __half22float2(ph);
+      const float e0 = s[t][u][0] - mnew + VWin<VC>::shift(2 * t);
+      const float e1 = s[t][u][1] - mnew + VWin<VC>::shift(2 * t + 1);
+      const float2 q = __half22float2(__floats2half2_rn(ex2_approx(e0), ex2_approx(e1)));
+      pf[t][u][0] = q.x;
+      pf[t][u][1] = q.y;
       if constexpr (VC == 0) {
-        ls += pf.x + pf.y;
+        ls += q.x + q.y;
       } else {
-        ls += pf.x * VWin<VC>::unshift(2 * t) + pf.y * VWin<VC>::unshift(2 * t + 1);
-        cs += pf.x + pf.y;
+        ls += q.x * VWin<VC>::unshift(2 * t) + q.y * VWin<VC>::unshift(2 * t + 1);
+        cs += q.x + q.y;
       }
-      const uint32_t pw = *reinterpret_cast<const uint32_t*>(&ph);
-      bv[t][nt][0] = movmatrix_t(pw & 0xffffu);
-      bv[t][nt][1] = movmatrix_t(pw >> 16);
     }
-    st.l[nt] = st.l[nt] * alpha[nt] + ls;
-    st.c[nt] = st.c[nt] * alpha[nt] + cs;
+    st.l[u] = st.l[u] * alpha[u] + ls;
+    st.c[u] = st.c[u] * alpha[u] + cs;
+  }
+  // B fragments of the V side: the 16 x 8 probability tile of token tile t in C-fragment
+  // layout (row t0 or t1, columns 2j, 2j+1), transposed by movmatrix.  The fp16 values are
+  // exact (they were rounded above).
+#pragma unroll
+  for (int t = 0; t < 8; ++t) {
+    const float c0 = pf[t][0][0], c1 = NG == 2 ? pf[t][NG - 1][0] : 0.f;
+    const float c2 = pf[t][0][1], c3 = NG == 2 ? pf[t][NG - 1][1] : 0.f;
+    bv[t][0] = movmatrix_t(pack_f16(c0, c1));
+    bv[t][1] = movmatrix_t(pack_f16(c2, c3));
   }
 }
 
 template <int G>
 __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs a) {
-  constexpr int NT = G / 4;
+  constexpr int NG = G / 4, NO = OAcc<G>::N;
   extern __shared__ __align__(128) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ring_bytes = a.ring_bytes;
   const size_t warp_bytes = (size_t)ring_bytes + decode_osm_bytes<G>();
   uint8_t* ring = smem + (size_t)warp * warp_bytes;
-  float4* osm = reinterpret_cast<float4*>(ring + ring_bytes);
+  float* osm = reinterpret_cast<float*>(ring + ring_bytes);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)kDecodeWarps * warp_bytes) + warp * kMaxStages;
   if (lane == 0) {
     for (int i = 0; i < kMaxStages; ++i) mbar_init(smem_addr(&bars[i]), 1);
@@ -391,16 +450,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     }
     WarpState<G> st;
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      st.m[nt] = -INFINITY;
-      st.l[nt] = 0.f;
-      st.c[nt] = 0.f;
+    for (int u = 0; u < NG; ++u) {
+      st.m[u] = -INFINITY;
+      st.l[u] = 0.f;
+      st.c[u] = 0.f;
     }
     const int nmu = ((vr >> 1) + 7) >> 3;
-    for (int k = 0; k < NT * nmu; ++k) {
-      const int nt = k / nmu, mu = k % nmu;
-      osm[(nt * 8 + mu) * 32 + lane] = make_float4(0.f, 0.f, 0.f, 0.f);
-    }
+    for (int k = 0; k < nmu * NO; ++k) osm[k * 32 + lane] = 0.f;
     // V window class (see row_softmax) and the factor 2^(10 - kmin) that turns the fed
     // products back into codes
     const int vc = (vr > 0 && vb <= 2) ? vb : 0;
@@ -410,9 +466,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
     const float* qhdr = reinterpret_cast<const float*>(qt);
     const uint2* bfrag = reinterpret_cast<const uint2*>(qt + kQtHeaderBytes);
-    float qsum[NT];
+    float qsum[NG];
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) qsum[nt] = qhdr[4 * nt + (lane & 3)];
+    for (int u = 0; u < NG; ++u) qsum[u] = qhdr[Heads<G>::head(lane & 3, u)];
     const float qscale = qhdr[8];
     const uint32_t one = a.one;
 
@@ -465,7 +521,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     };
 
     for (int row = row0; row < row1; ++row) {
-      float s[8][NT][2];
+      float s[8][NG][2];
       // ---- K row ----
       if (rbk) {
         const uint8_t* buf = acquire();
@@ -479,21 +535,21 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
 #pragma unroll
         for (int t = 0; t < 8; ++t)
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) s[t][nt][0] = s[t][nt][1] = 0.f;
+          for (int u = 0; u < NG; ++u) s[t][u][0] = s[t][u][1] = 0.f;
       }
       if ((row + 1) * kRowTokens > T) {  // only the last row of a sequence has masked tokens
         const int tbase = row * kRowTokens + (lane >> 2);
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
+        for (int u = 0; u < NG; ++u)
 #pragma unroll
           for (int t = 0; t < 8; ++t) {
-            if (tbase + 16 * t >= T) s[t][nt][0] = -INFINITY;
-            if (tbase + 16 * t + 8 >= T) s[t][nt][1] = -INFINITY;
+            if (tbase + 16 * t >= T) s[t][u][0] = -INFINITY;
+            if (tbase + 16 * t + 8 >= T) s[t][u][1] = -INFINITY;
           }
       }
-      uint32_t bv[8][NT][2];
+      uint32_t bv[8][2];
       bool rescale = false;
-      float alpha[NT];
+      float alpha[NG];
       if (vc == 1)
         row_softmax<G, 1>(s, st, alpha, rescale, bv);
       else if (vc == 2)
@@ -503,17 +559,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       // ---- V row ----
       if (rbv) {
         if (__any_sync(0xffffffffu, rescale)) {
+          for (int mu = 0; mu < nmu; ++mu) {
+            float* o = osm + (mu * 32 + lane) * NO;
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt)
-            for (int mu = 0; mu < nmu; ++mu) {
-              float4* o = osm + (nt * 8 + mu) * 32 + lane;
-              float4 v = *o;
-              v.x *= alpha[nt];
-              v.y *= alpha[nt];
-              v.z *= alpha[nt];
-              v.w *= alpha[nt];
-              *o = v;
-            }
+            for (int k = 0; k < NO; ++k) o[k] *= alpha[NG == 2 ? (k & 1) : 0];
+          }
         }
         const uint8_t* buf = acquire();
         if (!buf) {
@@ -528,8 +578,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     // ---- write the partial of this item ----
     __syncwarp();
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt) {
-      float l = st.l[nt], c = st.c[nt];
+    for (int u = 0; u < NG; ++u) {
+      float l = st.l[u], c = st.c[u];
       l += __shfl_xor_sync(0xffffffffu, l, 4);
       l += __shfl_xor_sync(0xffffffffu, l, 8);
       l += __shfl_xor_sync(0xffffffffu, l, 16);
@@ -537,17 +587,19 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       c += __shfl_xor_sync(0xffffffffu, c, 8);
       c += __shfl_xor_sync(0xffffffffu, c, 16);
       if (vc == 0) c = l;
-      const int g = 4 * nt + (lane & 3);
+      const int g = Heads<G>::head(lane & 3, u);
       float* pg = part + g * gstride;
       if ((lane >> 2) == 0) {
-        pg[0] = st.m[nt];
+        pg[0] = st.m[u];
         pg[1] = l;
       }
       for (int mu = 0; mu < nmu; ++mu) {
-        const float4 v = osm[(nt * 8 + mu) * 32 + lane];
+        const float* o = osm + (mu * 32 + lane) * NO;
+        // G = 4: [ch0, ch1]; G = 8: [ch0 head 2j, ch0 head 2j+1, ch1 head 2j, ch1 head 2j+1]
+        const float o0 = NO == 2 ? o[0] : o[u], o1 = NO == 2 ? o[1] : o[2 + u];
         const int ch0 = 16 * mu + (lane >> 2), ch1 = ch0 + 8;
-        if (ch0 < vr) pg[4 + ch0] = ((v.x + v.y) - c) * vout;
-        if (ch1 < vr) pg[4 + ch1] = ((v.z + v.w) - c) * vout;
+        if (ch0 < vr) pg[4 + ch0] = (o0 - c) * vout;
+        if (ch1 < vr) pg[4 + ch1] = (o1 - c) * vout;
       }
     }
     __syncwarp();

@@ -123,6 +123,8 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
 }
 
 namespace {
+size_t decode_osm_bytes_host(int G) { return (size_t)8 * 32 * (G == 4 ? 2 : 4) * sizeof(float); }
+
 enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
 template <int G>
@@ -132,7 +134,7 @@ cobra_status launch_decode(const DecodeArgs& a, int n_groups, int n_items, int s
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kScan) {
-    const size_t smem = (size_t)kDecodeWarps * ((size_t)a.ring_bytes + (size_t)(G / 4) * 8 * 32 * 16 + kMaxStages * 8);
+    const size_t smem = (size_t)kDecodeWarps * ((size_t)a.ring_bytes + decode_osm_bytes_host(G) + kMaxStages * 8);
     static size_t attr_set = 0;
     if (smem > attr_set) {
       if (cudaFuncSetAttribute(decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
