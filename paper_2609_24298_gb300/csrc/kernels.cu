@@ -1,5 +1,6 @@
 // libcobra device entry points: argument checks and launches for compress, append and
 // decode attention, plus the device status check.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -9,6 +10,7 @@
 #include "../../include/cobra.h"
 #include "common.cuh"
 #include "compress.cuh"
+#include "compress_tc.cuh"
 #include "decode.cuh"
 
 using namespace cobra;
@@ -39,6 +41,65 @@ int sm_count() {
 
 }  // namespace
 
+namespace {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 5-D tensor map over x (bf16): dimension 0 = the 128 head dims (contiguous), the other four
+// (kv head, token, sequence, layer) ordered by increasing stride as the TMA unit requires.
+// Box: 64 dims x 128 tokens, 128-byte swizzle; tokens past n_tok read as zeros.
+cobra_status make_x_map(const cobra_compress_desc* d, const void* x, int n_tok, CUtensorMap* map, int slots[4]) {
+  EncodeTiledFn enc = encode_tiled();
+  if (!enc) return COBRA_ECUDA;
+  struct Dim {
+    long long size, stride_bytes;
+    int box, logical;
+  };
+  Dim dims[4] = {{d->n_kv_heads, d->x_stride_head * 2, 1, 0},
+                 {n_tok, d->x_stride_tok * 2, kRowTokens, 1},
+                 {d->n_seqs, d->x_stride_seq * 2, 1, 2},
+                 {d->n_layers, d->x_stride_layer * 2, 1, 3}};
+  // a dimension of size 1 is never stepped: give it a stride that keeps the order valid
+  long long run = 256;
+  for (int pass = 0; pass < 4; ++pass)
+    for (auto& e : dims)
+      if (e.size > 1) run = std::max(run, e.stride_bytes * e.size);
+  for (auto& e : dims)
+    if (e.size == 1) e.stride_bytes = run;
+  std::stable_sort(dims, dims + 4, [](const Dim& p, const Dim& q) { return p.stride_bytes < q.stride_bytes; });
+  cuuint64_t gdim[5] = {(cuuint64_t)kD, 0, 0, 0, 0};
+  cuuint64_t gstride[4];
+  cuuint32_t box[5] = {64, 1, 1, 1, 1};
+  cuuint32_t estride[5] = {1, 1, 1, 1, 1};
+  for (int i = 0; i < 4; ++i) {
+    if (dims[i].stride_bytes <= 0 || dims[i].stride_bytes % 16 || dims[i].size < 1) return COBRA_EINVAL;
+    gdim[i + 1] = (cuuint64_t)dims[i].size;
+    gstride[i] = (cuuint64_t)dims[i].stride_bytes;
+    box[i + 1] = (cuuint32_t)dims[i].box;
+    slots[dims[i].logical] = i + 1;
+  }
+  const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(x), gdim, gstride, box, estride,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? COBRA_OK : COBRA_EINVAL;
+}
+
+}  // namespace
+
 extern "C" cobra_status cobra_compress(const void* params, const cobra_compress_desc* d, const void* x, int t0, int n_tok,
                                        uint8_t* cache, const int* page_table, void* stream) {
   cobra_status st = check_compress_desc(d);
@@ -54,24 +115,23 @@ extern "C" cobra_status cobra_compress(const void* params, const cobra_compress_
     return COBRA_EINVAL;
   }
   if (n_tok == 0) return COBRA_OK;
+  CUtensorMap map;
+  int slots[4];
+  st = make_x_map(d, x, n_tok, &map, slots);
+  if (st != COBRA_OK) return st;
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(compress_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kCompressSmem) != cudaSuccess)
+    if (cudaFuncSetAttribute(compress_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmemBytes) !=
+        cudaSuccess)
       return COBRA_ECUDA;
     attr = true;
   }
-  CompressArgs a{};
+  TcArgs a{};
   a.block = static_cast<const unsigned char*>(params);
-  a.x = static_cast<const __nv_bfloat16*>(x);
   a.cache = cache;
   a.page_table = page_table;
-  a.sl = d->x_stride_layer;
-  a.ss = d->x_stride_seq;
-  a.st = d->x_stride_tok;
-  a.sh = d->x_stride_head;
   a.head0 = d->head0;
   a.layer_stride = d->layer_stride;
-  a.n_layers = d->n_layers;
   a.n_kv = d->n_kv_heads;
   a.side = d->side;
   a.n_seqs = d->n_seqs;
@@ -79,15 +139,19 @@ extern "C" cobra_status cobra_compress(const void* params, const cobra_compress_
   a.pages_per_seq = d->pages_per_seq;
   a.t0 = t0;
   a.n_tok = n_tok;
-  const int heads = d->n_layers * d->n_kv_heads;
+  a.slot_head = slots[0];
+  a.slot_tok = slots[1];
+  a.slot_seq = slots[2];
+  a.slot_layer = slots[3];
+  const long long heads = (long long)d->n_layers * d->n_kv_heads;
   const long long tiles = (long long)d->n_seqs * ((n_tok + kRowTokens - 1) / kRowTokens);
-  // about two waves of CTAs, each CTA converting its head's basis once
-  long long chunks = std::max(1LL, (2LL * sm_count() + heads - 1) / heads);
+  // one CTA per SM: about one wave of CTAs, each converting its head's basis once
+  long long chunks = std::max(1LL, (sm_count() + heads - 1) / heads);
   chunks = std::min(chunks, tiles);
   a.chunks = (int)chunks;
-  const long long grid = (long long)heads * chunks;
+  const long long grid = heads * chunks;
   if (grid > 0x7fffffffLL) return COBRA_EINVAL;
-  compress_kernel<<<(unsigned)grid, kCompressThreads, kCompressSmem, (cudaStream_t)stream>>>(a);
+  compress_tc_kernel<<<(unsigned)grid, kTcThreads, kTcSmemBytes, (cudaStream_t)stream>>>(map, a);
   return launch_status();
 }
 

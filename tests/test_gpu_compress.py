@@ -136,3 +136,32 @@ def test_append_matches_compress(side):
     for q in range(seqs):
         for h, p in enumerate(params):
             check_head(host, offs[h], side, p, xs[q, :, h], T + extra, seq=q, rows_per_seq=nrows)
+
+
+def test_compress_head_major_layers_padded_tokens():
+    """x stored [layer][head][seq][token][136] (head-major, 8 padding elements per token):
+    the tensor-map dimensions are ordered by stride, not by the descriptor's field order."""
+    L, H, seqs, T, dpad = 2, 3, 2, 300, 136
+    srcs = [synth.HeadSource(16, l, h, 0, (0.3, 2.5)) for l in range(L) for h in range(H)]
+    rbs = [(128, 2), (40, 4), (22, 7), (64, 1), (90, 3), (128, 5)]
+    params = [oracle_head(s, r, b) for s, (r, b) in zip(srcs, rbs)]
+    nrows = -(-T // 128)
+    block, offs, total, r, b = upload(params, seqs * nrows)
+    cache = torch.zeros(total, dtype=torch.uint8, device=DEV)
+    xs = np.zeros((L, H, seqs, T, dpad), np.float32)
+    for l in range(L):
+        for h in range(H):
+            for q in range(seqs):
+                xs[l, h, q, :, :128] = srcs[l * H + h].tokens(T, seq=q)
+    x = torch.tensor(xs, dtype=torch.bfloat16, device=DEV)
+    desc = cobra.compress_desc(head0=0, layer_stride=H, n_layers=L, n_kv_heads=H, side=0, n_seqs=seqs,
+                               rows_per_seq=nrows, x_stride_layer=H * seqs * T * dpad, x_stride_seq=T * dpad,
+                               x_stride_tok=dpad, x_stride_head=seqs * T * dpad)
+    cobra.cobra_compress(block, desc, x, 0, T, cache)
+    assert cobra.cobra_check() == cobra.COBRA_OK
+    host = cache.cpu().numpy()
+    for l in range(L):
+        for h in range(H):
+            for q in range(seqs):
+                check_head(host, offs[l * H + h], 0, params[l * H + h], xs[l, h, q, :, :128], T, seq=q,
+                           rows_per_seq=nrows)
