@@ -48,6 +48,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="oracle sample budget for cpu_baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None, help="fewer layers (profiling runs only)")
+    ap.add_argument("--no-compress", action="store_true", help="skip the prefill compress measurement")
+    ap.add_argument("--compress-only", action="store_true", help="only the prefill compress measurement")
+    ap.add_argument("--compress-layers", type=int, default=None, help="fewer layers (profiling runs only)")
     return ap.parse_args()
 
 
@@ -229,6 +232,78 @@ def workload_config(spec):
 
 
 # ---------------------------------------------------------------------------------------
+# prefill compress (the tensor-core projection path)
+# ---------------------------------------------------------------------------------------
+COMPRESS_CFG = 4
+
+
+def run_compress_leg(args, dev, stream, peak):
+    """Compress every token of the prefill workload - 32 layers x 8 kv heads x batch 64 x 4096
+    tokens of bf16 K and V at 4 bpd - from inputs resident in HBM (about 34 GB, far larger
+    than L2), one cobra_compress launch per side covering all layers.  Returns the JSON
+    object reported under "compress"."""
+    import torch
+
+    from paper_2609_24298_gb300 import cobra, pipeline, synth
+
+    spec = synth.CONFIGS[COMPRESS_CFG]
+    L, H, S, T = spec["layers"], spec["kv_heads"], spec["seqs"], spec["tokens"]
+    if args.compress_layers:
+        L = args.compress_layers
+    hp, srcs = pipeline.build_params(COMPRESS_CFG, L, spec["bpd"], joint=False)
+    rows = -(-T // 128)
+    dp = pipeline.DeviceParams(hp, S * rows, device=dev)
+    xs = []
+    for side in (0, 1):
+        x = torch.empty((L, S, T, H, 128), dtype=torch.bfloat16, device=dev)
+        for l in range(L):
+            x[l] = pipeline.device_tokens([srcs[side * L * H + l * H + h] for h in range(H)], S, T,
+                                          seed=COMPRESS_CFG * 1000003 + 2 * l + side, device=dev)
+        xs.append(x)
+    descs = [cobra.compress_desc(head0=side * L * H, layer_stride=H, n_layers=L, n_kv_heads=H, side=side, n_seqs=S,
+                                 rows_per_seq=rows, x_stride_layer=S * T * H * 128, x_stride_seq=T * H * 128,
+                                 x_stride_tok=H * 128, x_stride_head=128) for side in (0, 1)]
+
+    def one_pass():
+        for side in (0, 1):
+            cobra.cobra_compress(dp.block, descs[side], xs[side], 0, T, dp.cache, None, stream)
+
+    for _ in range(3):
+        one_pass()
+    torch.cuda.synchronize()
+    if cobra.cobra_check(stream) != cobra.COBRA_OK:
+        raise RuntimeError("device status after compress warm-up")
+    K = max(5, min(50, args.steps // 40))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(K):
+        one_pass()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if cobra.cobra_check(stream) != cobra.COBRA_OK:
+        raise RuntimeError("device status after the compress timed region")
+    ms = e0.elapsed_time(e1) / K
+    in_bytes = 2 * L * S * T * H * 128 * 2
+    out_bytes = int(sum(16 * int(r) * int(b) for r, b in zip(hp.r, hp.b) if r > 0)) * S * rows
+    flops = 2 * 128 * int(sum(int(r) for r in hp.r)) * S * T  # algorithmic y = W^T x per token-head
+    gbs = (in_bytes + out_bytes) / (ms * 1e-3) / 1e9
+    tokens = S * T
+    del xs
+    return {
+        "metric": "compress tok/s", "value": tokens / (ms * 1e-3), "unit": "tok/s",
+        "workload": f"prefill compress: {L} layers x {H} kv heads x batch {S} x {T} tokens of bf16 K and V "
+                    f"(head_dim 128) at {spec['bpd']:g} bpd, inputs resident in HBM",
+        "tokens_per_pass": tokens, "head_tokens_per_s": tokens * L * H * 2 / (ms * 1e-3), "ms_per_pass": ms,
+        "passes": K, "launches": 2 * K, "gbs": gbs,
+        "roofline": {"bound": "hbm", "kernel": "compress_tc_kernel", "achieved": gbs, "peak": peak, "unit": "GB/s",
+                     "frac": gbs / peak, "algorithmic_bytes_per_pass": in_bytes + out_bytes, "traffic": None,
+                     "tensor_tflops_algorithmic": flops / (ms * 1e-3) / 1e12},
+        "l2": "inputs larger than L2 (about 34 GB of bf16 K/V read every pass)",
+    }
+
+
+# ---------------------------------------------------------------------------------------
 # the CUDA path
 # ---------------------------------------------------------------------------------------
 def run_cobra(args):
@@ -251,6 +326,9 @@ def run_cobra(args):
     G = spec["q_heads"] // H
     Hq = H * G
     cobra.lib()
+    if args.compress_only:
+        print(json.dumps(run_compress_leg(args, dev, torch.cuda.current_stream(), hbm_peak()[0])), flush=True)
+        return
 
     # cpu baseline first, before any GPU work (rank 0, N = 1 only)
     cpu = None
@@ -373,6 +451,10 @@ def run_cobra(args):
 
     peak, peak_kind = hbm_peak()
     achieved = bytes_step / (scan_ms * 1e-3) / 1e9
+    compress = None
+    if not args.no_compress:
+        del hk, hv, hq, hout
+        compress = run_compress_leg(args, dev, stream, peak)
     traffic = profiled_traffic()
     if rank == 0:
         line = {
@@ -385,6 +467,7 @@ def run_cobra(args):
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic, "scan_ms": scan_ms,
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
+            "compress": compress,
             "cpu_baseline": cpu,
             "e2e": {"value": bytes_step * world / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},

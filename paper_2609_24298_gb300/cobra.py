@@ -118,6 +118,11 @@ def _ptr(x):
         return None
     if isinstance(x, int):
         return x
+    if not x.is_contiguous():
+        # the library addresses buffers through the strides in its descriptors, which refer
+        # to the memory itself: a permuted or sliced view would be read with the wrong layout
+        raise ValueError("device tensors passed to libcobra must be contiguous; describe other layouts "
+                         "with the descriptor strides over a contiguous buffer")
     return x.data_ptr()
 
 

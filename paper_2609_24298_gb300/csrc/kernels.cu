@@ -145,9 +145,21 @@ extern "C" cobra_status cobra_compress(const void* params, const cobra_compress_
   a.slot_layer = slots[3];
   const long long heads = (long long)d->n_layers * d->n_kv_heads;
   const long long tiles = (long long)d->n_seqs * ((n_tok + kRowTokens - 1) / kRowTokens);
-  // one CTA per SM: about one wave of CTAs, each converting its head's basis once
-  long long chunks = std::max(1LL, (sm_count() + heads - 1) / heads);
-  chunks = std::min(chunks, tiles);
+  // One CTA per SM at a time.  Split each head's tiles into the number of chunks that fills
+  // whole waves of SMs best (the last wave of a ragged grid idles SMs), keeping at least 16
+  // tiles per CTA so that converting the head's basis stays a small part of its work.
+  const long long sms = sm_count();
+  const long long cmax = std::max(1LL, std::min(tiles / 16, 8 * sms));
+  long long chunks = 1;
+  double best = -1.0;
+  for (long long c = 1; c <= cmax; ++c) {
+    const long long total = heads * c, waves = (total + sms - 1) / sms;
+    const double eff = (double)total / (double)(waves * sms);
+    if (eff > best + 1e-9) {
+      best = eff;
+      chunks = c;
+    }
+  }
   a.chunks = (int)chunks;
   const long long grid = heads * chunks;
   if (grid > 0x7fffffffLL) return COBRA_EINVAL;

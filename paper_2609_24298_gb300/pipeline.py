@@ -125,8 +125,8 @@ def device_tokens(src_list, n_seqs: int, n_tok: int, seed: int, device="cuda", t
     gen = torch.Generator(device=device)
     gen.manual_seed(seed)
     g = torch.randn((n_seqs, n_tok, len(src_list), D), generator=gen, device=device, dtype=torch.float32)
-    x = torch.einsum("sthd,hed->sthe", g, A)
-    return x.to(torch.bfloat16)
+    x = torch.einsum("sthd,hed->sthe", g, A)  # einsum may return a permuted layout
+    return x.to(torch.bfloat16).contiguous()
 
 
 def fill_cache(wl: Workload, srcs, device="cuda", stream=None, keep_layers=()):

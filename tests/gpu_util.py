@@ -20,9 +20,10 @@ def oracle_head(src, r, b, q_cal=None):
     return ocal.head_params(cal, r, b, synth.hadamard_signs(*src.key)) | {"w": cal["w"]}
 
 
-def oracle_heads_allocated(cfg, layers, bpd, joint=False):
-    """Oracle calibration + allocation + fusion for every (side, layer, kv head) of a config.
-    Returns (params list in library head order [K heads..., V heads...], sources)."""
+def oracle_calibrations(cfg, layers, joint=False):
+    """Oracle calibration of every (side, layer, kv head) of a config, in library head order
+    [K heads..., V heads...]; KL weights with the config's calibration queries for separate
+    K allocation, MSE weights otherwise.  Returns (calibrations, sources)."""
     spec = synth.CONFIGS[cfg]
     H = spec["kv_heads"]
     G = spec["q_heads"] // H
@@ -33,17 +34,28 @@ def oracle_heads_allocated(cfg, layers, bpd, joint=False):
         l, h = divmod(rem, H)
         q = synth.calibration_queries(cfg, l, h, G, 512, spec["alpha"]) if (side == 0 and not joint) else None
         cals.append(ocal.calibrate_head(s.calibration(512), q))
+    return cals, srcs
+
+
+def oracle_allocated_params(cals, srcs, bpd, joint=False):
+    """Oracle allocation at `bpd` (K and V separately, or jointly) and basis fusion."""
     w = np.stack([c["w"] for c in cals])
-    n = layers * H
+    n = len(cals) // 2
     if joint:
         res = oal.allocate(w, bpd)
         r, b = res["r"], res["b"]
     else:
         a, c = oal.allocate(w[:n], bpd), oal.allocate(w[n:], bpd)
         r, b = np.concatenate([a["r"], c["r"]]), np.concatenate([a["b"], c["b"]])
-    params = [ocal.head_params(c, int(rr), int(bb) if rr else 1, synth.hadamard_signs(*s.key))
-              for c, s, rr, bb in zip(cals, srcs, r, b)]
-    return params, srcs
+    return [ocal.head_params(c, int(rr), int(bb) if rr else 1, synth.hadamard_signs(*s.key))
+            for c, s, rr, bb in zip(cals, srcs, r, b)]
+
+
+def oracle_heads_allocated(cfg, layers, bpd, joint=False):
+    """Oracle calibration + allocation + fusion for every (side, layer, kv head) of a config.
+    Returns (params list in library head order [K heads..., V heads...], sources)."""
+    cals, srcs = oracle_calibrations(cfg, layers, joint)
+    return oracle_allocated_params(cals, srcs, bpd, joint), srcs
 
 
 def upload(params, n_slots):
@@ -86,3 +98,14 @@ def rel_err(o, ref):
     """max over query heads of ||o - ref||_inf / ||ref||_inf."""
     den = np.maximum(np.abs(ref).max(axis=-1), 1e-30)
     return float((np.abs(o - ref).max(axis=-1) / den).max())
+
+
+def oracle_head_params(params):
+    """The oracle's per-head parameters in the product's HeadParams form (for DeviceParams)."""
+    from paper_2609_24298_gb300 import pipeline
+    r = np.array([p["r"] for p in params], np.int32)
+    b = np.array([p["b"] if p["r"] else 1 for p in params], np.int32)
+    delta = np.array([p["delta"] if p["r"] else 0.0 for p in params], np.float32)
+    mu = np.stack([p["mu"] for p in params]).astype(np.float32)
+    return pipeline.HeadParams(r, b, delta, [p["W"] for p in params], mu)
+

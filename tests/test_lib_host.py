@@ -174,3 +174,13 @@ def test_decode_plan_sizes(L):
     b = np.array([2, 3, 8, 0], np.int32)
     n = cobra.cobra_decode_workspace_size(dd, r, b, np.array([32768, 1, 0], np.int32))
     assert n > 0 and n % 256 == 0
+
+
+def test_binding_rejects_non_contiguous_buffers():
+    import torch
+    x = torch.zeros((4, 6))
+    assert cobra._ptr(x) == x.data_ptr()
+    with pytest.raises(ValueError):
+        cobra._ptr(x.t())
+    with pytest.raises(ValueError):
+        cobra._ptr(x[:, ::2])
