@@ -54,24 +54,33 @@ def parse_args():
     return ap.parse_args()
 
 
-def scan_source_hash() -> str:
+COMPRESS_PROFILE = os.path.join(ROOT, "profiles", "compress_tc_prefill_4bpd.txt")
+COMPRESS_SOURCES = ["paper_2609_24298_gb300/csrc/compress_tc.cuh", "paper_2609_24298_gb300/csrc/compress.cuh",
+                    "paper_2609_24298_gb300/csrc/common.cuh"]
+
+
+def source_hash(sources) -> str:
     h = hashlib.sha256()
-    for p in SCAN_SOURCES:
+    for p in sources:
         with open(os.path.join(ROOT, p), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per scan launch from the committed ncu summary, if it was taken on the
-    current kernel source (else None)."""
+def scan_source_hash() -> str:
+    return source_hash(SCAN_SOURCES)
+
+
+def profiled_traffic(profile=PROFILE, sources=SCAN_SOURCES):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on the current
+    kernel source (else None)."""
     try:
-        txt = open(PROFILE).read()
+        txt = open(profile).read()
     except OSError:
         return None
     m1 = re.search(r"traffic_bytes_per_launch\s*=\s*([0-9.eE+]+)", txt)
     m2 = re.search(r"kernel_source_sha\s*=\s*([0-9a-f]+)", txt)
-    if not m1 or not m2 or m2.group(1) != scan_source_hash():
+    if not m1 or not m2 or m2.group(1) != source_hash(sources):
         return None
     return float(m1.group(1))
 
@@ -284,6 +293,7 @@ def run_compress_leg(args, dev, stream, peak):
     if cobra.cobra_check(stream) != cobra.COBRA_OK:
         raise RuntimeError("device status after the compress timed region")
     ms = e0.elapsed_time(e1) / K
+    traffic = profiled_traffic(COMPRESS_PROFILE, COMPRESS_SOURCES)
     in_bytes = 2 * L * S * T * H * 128 * 2
     out_bytes = int(sum(16 * int(r) * int(b) for r, b in zip(hp.r, hp.b) if r > 0)) * S * rows
     flops = 2 * 128 * int(sum(int(r) for r in hp.r)) * S * T  # algorithmic y = W^T x per token-head
@@ -297,9 +307,10 @@ def run_compress_leg(args, dev, stream, peak):
         "tokens_per_pass": tokens, "head_tokens_per_s": tokens * L * H * 2 / (ms * 1e-3), "ms_per_pass": ms,
         "passes": K, "launches": 2 * K, "gbs": gbs,
         "roofline": {"bound": "hbm", "kernel": "compress_tc_kernel", "achieved": gbs, "peak": peak, "unit": "GB/s",
-                     "frac": gbs / peak, "algorithmic_bytes_per_pass": in_bytes + out_bytes, "traffic": None,
+                     "frac": gbs / peak, "algorithmic_bytes_per_pass": in_bytes + out_bytes,
+                     "traffic_per_launch": traffic if L == 32 else None,
                      "tensor_tflops_algorithmic": flops / (ms * 1e-3) / 1e12},
-        "l2": "inputs larger than L2 (about 34 GB of bf16 K/V read every pass)",
+        "l2": f"inputs larger than L2 ({in_bytes / 1e9:.1f} GB of bf16 K/V read every pass)",
     }
 
 
