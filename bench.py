@@ -374,16 +374,27 @@ def run_cobra(args):
                                  x_stride_head=128) for side in (0, 1)]
     block, cache = wl.dev.block, wl.dev.cache
 
-    def step(ev_scan0=None, ev_scan1=None):
+    stages = ("append_k", "append_v", "qproj", "scan", "combine")
+
+    def step(ev=None):
+        # ev: 6 events bracketing the 5 launches (recorded on the launch stream)
+        if ev is not None:
+            ev[0].record(stream)
         cobra.cobra_append(block, adesc[0], xk, pos, cache, None, stream)
+        if ev is not None:
+            ev[1].record(stream)
         cobra.cobra_append(block, adesc[1], xv, pos, cache, None, stream)
+        if ev is not None:
+            ev[2].record(stream)
         cobra.cobra_decode_qproj(block, desc, info, q, ws, nbytes_ws, stream)
-        if ev_scan0 is not None:
-            ev_scan0.record(stream)
+        if ev is not None:
+            ev[3].record(stream)
         cobra.cobra_decode_scan(block, desc, info, cache, lens, None, ws, nbytes_ws, stream)
-        if ev_scan1 is not None:
-            ev_scan1.record(stream)
+        if ev is not None:
+            ev[4].record(stream)
         cobra.cobra_decode_combine(block, desc, info, lens, out, ws, nbytes_ws, stream)
+        if ev is not None:
+            ev[5].record(stream)
 
     launches_per_step = 5
     for _ in range(args.warmup):
@@ -395,7 +406,7 @@ def run_cobra(args):
 
     # timed region: the whole steps, and the scan kernel alone (events on the launch stream)
     K = args.steps
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(K)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     if world > 1:
@@ -405,14 +416,15 @@ def run_cobra(args):
     time.sleep(0.3)
     t_start.record(stream)
     for k in range(K):
-        step(ev[k][0], ev[k][1])
+        step(ev[k])
     t_end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
     if world > 1:
         dist.barrier()
     total_ms = t_start.elapsed_time(t_end)
-    scan_ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+    stage_ms = {name: float(np.mean([e[i].elapsed_time(e[i + 1]) for e in ev])) for i, name in enumerate(stages)}
+    scan_ms = stage_ms["scan"]
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -482,6 +494,7 @@ def run_cobra(args):
             "cpu_baseline": cpu,
             "e2e": {"value": bytes_step * world / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "stage_ms": stage_ms,
             "gpu_launches": launches_per_step * K,
             "clocks": clk,
         }

@@ -196,6 +196,29 @@ __device__ __forceinline__ void load_piece_or_zero(const uint8_t* p, bool valid,
   }
 }
 
+// 16-byte global -> shared copies that stay in flight until cp_async_wait_all.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+
+// Rows [0, r) of a basis (fp32, 128 per row, 16-byte aligned) into shared memory with row
+// stride ld floats (a multiple of 4); rows [r, 128) are zeroed.  Every copy is issued before
+// any is waited for.  The caller synchronises the block before reading.
+__device__ __forceinline__ void stage_basis(const float* W, int r, int ld, float* dst) {
+  for (int idx = threadIdx.x; idx < 128 * 32; idx += blockDim.x) {
+    const int i = idx >> 5, c = idx & 31;
+    float* d = dst + (size_t)i * ld + 4 * c;
+    if (i < r)
+      cp_async16(smem_addr(d), W + (size_t)idx * 4);
+    else
+      *reinterpret_cast<float4*>(d) = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  cp_async_wait_all();
+}
+
 // ---------------------------------------------------------------------------------------
 // parameter block access
 // ---------------------------------------------------------------------------------------

@@ -64,66 +64,97 @@ __device__ __forceinline__ void pack_piece(const uint8_t* codes, int ldc, int si
   for (int k = 0; k < B; ++k) dst[k] = w[k];
 }
 
-// a8: single-token append.  One warp per (layer, kv head, sequence).
-__global__ void __launch_bounds__(128) append_kernel(CompressArgs a) {
-  __shared__ float xs[4][kD];
+// a8: single-token append.  One CTA of 8 warps per (layer, kv head): the head's basis is staged
+// in shared memory once (row stride kAppendWLd floats, so that a warp's 16-byte row reads are
+// conflict-free) and each warp appends the token of one sequence at a time.
+constexpr int kAppendThreads = 256;
+constexpr int kAppendWLd = 132;
+__host__ __device__ constexpr size_t append_smem_bytes() {
+  return sizeof(float) * ((size_t)kD * kAppendWLd + (size_t)(kAppendThreads / 32) * kD + kD);
+}
+
+__global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) {
+  extern __shared__ __align__(16) float apsm[];
+  float* Ws = apsm;                     // [kD][kAppendWLd]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const long long gw = (long long)blockIdx.x * 4 + warp;
-  const long long total = (long long)a.n_layers * a.n_kv * a.n_seqs;
-  if (gw >= total) return;
-  const int seq = (int)(gw % a.n_seqs);
-  const int kv = (int)((gw / a.n_seqs) % a.n_kv);
-  const int layer = (int)(gw / ((long long)a.n_seqs * a.n_kv));
+  float* wmu = Ws + kD * kAppendWLd + (kAppendThreads / 32) * kD;  // W^T mu
+  float* xs = Ws + kD * kAppendWLd + warp * kD;
+  const int layer = blockIdx.x / a.n_kv, kv = blockIdx.x % a.n_kv;
   const HeadEntry he = head_table(a.block)[a.head0 + layer * a.layer_stride + kv];
   const int r = he.r, b = he.b;
-  const __nv_bfloat16* xp = a.x + layer * a.sl + seq * a.ss + kv * a.sh;
-#pragma unroll
-  for (int k = 0; k < 4; ++k) xs[warp][lane + 32 * k] = __bfloat162float(xp[lane + 32 * k]);
-  __syncwarp();
   if (r == 0) return;
-  const int p = a.pos[seq];
-  const int row = p >> 7, tt = p & 127;
-  const bool in_range = p >= 0 && (a.page_table ? (row >> 1) < a.pages_per_seq : row < a.rows_per_seq);
-  if (!in_range) {  // a position past the cache's capacity is never written
-    if (lane == 0) atomicOr(&g_status, 2u);
-    return;
-  }
-  const uint32_t rb = 16u * r * b;
-  uint8_t* rowp = a.cache + row_offset(he.cache_off, rb, seq, row, a.page_table, a.pages_per_seq, a.rows_per_seq);
   const float* pool = param_pool(a.block);
+  // the first sequence's token and position are loaded while the basis is staged
+  __nv_bfloat16 xr[4];
+  int p_next = 0;
+  if (warp < a.n_seqs) {
+    const __nv_bfloat16* xp = a.x + layer * a.sl + warp * a.ss + kv * a.sh;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) xr[k] = xp[lane + 32 * k];
+    p_next = a.pos[warp];
+  }
+  // W^T mu holds r floats (the pool is padded to 32 floats, so whole 16-byte chunks stay in it)
+  if (threadIdx.x < (r + 3) / 4) cp_async16(smem_addr(wmu + 4 * threadIdx.x), pool + he.wmu_off + 4 * threadIdx.x);
+  stage_basis(pool + he.w_off, r, kAppendWLd, Ws);
+  __syncthreads();
+  const uint32_t rb = 16u * r * b;
   const float inv_delta = he.inv_delta, half = (float)(1 << (b - 1));
   const int cmax = (1 << b) - 1;
-  const int tau = tt >> 4, t16 = tt & 15, rho = 2 * tau + (t16 >> 3);
-  for (int i = lane; i < r; i += 32) {
-    const float* w = pool + he.w_off + (size_t)i * kD;
-    float y = 0.f;
-    for (int dd = 0; dd < kD; dd += 4) {
-      const float4 wv = *reinterpret_cast<const float4*>(w + dd);
-      y += wv.x * xs[warp][dd] + wv.y * xs[warp][dd + 1] + wv.z * xs[warp][dd + 2] + wv.w * xs[warp][dd + 3];
+  for (int seq = warp; seq < a.n_seqs; seq += kAppendThreads / 32) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) xs[lane + 32 * k] = __bfloat162float(xr[k]);
+    const int p = p_next;
+    // the next sequence's token and position, in flight during this one's projection
+    const int nseq = seq + kAppendThreads / 32;
+    if (nseq < a.n_seqs) {
+      const __nv_bfloat16* xp = a.x + layer * a.sl + nseq * a.ss + kv * a.sh;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) xr[k] = xp[lane + 32 * k];
+      p_next = a.pos[nseq];
     }
-    y -= pool[he.wmu_off + i];
-    int code = (int)floorf(fmaf(y, inv_delta, half));
-    code = code < 0 ? 0 : (code > cmax ? cmax : code);
-    int piece, h;
-    if (a.side == 0) {
-      piece = t16 & 7;
-      h = i & 1;
-    } else {
-      piece = 4 * (i & 1) + ((t16 >> 1) & 3);
-      h = t16 & 1;
+    __syncwarp();
+    const int row = p >> 7, tt = p & 127;
+    const bool in_range = p >= 0 && (a.page_table ? (row >> 1) < a.pages_per_seq : row < a.rows_per_seq);
+    if (!in_range) {  // a position past the cache's capacity is never written
+      if (lane == 0) atomicOr(&g_status, 2u);
+      __syncwarp();
+      continue;
     }
-    uint32_t* words = reinterpret_cast<uint32_t*>(rowp + (i >> 1) * 32 * b + piece * 4 * b);
-    const int x0 = rho * b;
-    const int w0 = x0 >> 4, o0 = x0 & 15;
-    const int n0 = min(b, 16 - o0);
-    const uint32_t m0 = ((1u << n0) - 1u) << (16 * h + o0);
-    atomicAnd(words + w0, ~m0);
-    atomicOr(words + w0, ((uint32_t)code << (16 * h + o0)) & m0);
-    if (n0 < b) {
-      const uint32_t m1 = ((1u << (b - n0)) - 1u) << (16 * h);
-      atomicAnd(words + w0 + 1, ~m1);
-      atomicOr(words + w0 + 1, ((uint32_t)code >> n0) << (16 * h) & m1);
+    uint8_t* rowp = a.cache + row_offset(he.cache_off, rb, seq, row, a.page_table, a.pages_per_seq, a.rows_per_seq);
+    const int tau = tt >> 4, t16 = tt & 15, rho = 2 * tau + (t16 >> 3);
+    for (int i = lane; i < r; i += 32) {
+      const float* w = Ws + i * kAppendWLd;
+      float y = 0.f;
+      for (int dd = 0; dd < kD; dd += 4) {
+        const float4 wv = *reinterpret_cast<const float4*>(w + dd);
+        const float4 xv = *reinterpret_cast<const float4*>(xs + dd);
+        y += wv.x * xv.x + wv.y * xv.y + wv.z * xv.z + wv.w * xv.w;
+      }
+      y -= wmu[i];
+      int code = (int)floorf(fmaf(y, inv_delta, half));
+      code = code < 0 ? 0 : (code > cmax ? cmax : code);
+      int piece, h;
+      if (a.side == 0) {
+        piece = t16 & 7;
+        h = i & 1;
+      } else {
+        piece = 4 * (i & 1) + ((t16 >> 1) & 3);
+        h = t16 & 1;
+      }
+      uint32_t* words = reinterpret_cast<uint32_t*>(rowp + (i >> 1) * 32 * b + piece * 4 * b);
+      const int x0 = rho * b;
+      const int w0 = x0 >> 4, o0 = x0 & 15;
+      const int n0 = min(b, 16 - o0);
+      const uint32_t m0 = ((1u << n0) - 1u) << (16 * h + o0);
+      atomicAnd(words + w0, ~m0);
+      atomicOr(words + w0, ((uint32_t)code << (16 * h + o0)) & m0);
+      if (n0 < b) {
+        const uint32_t m1 = ((1u << (b - n0)) - 1u) << (16 * h);
+        atomicAnd(words + w0 + 1, ~m1);
+        atomicOr(words + w0 + 1, ((uint32_t)code >> n0) << (16 * h) & m1);
+      }
     }
+    __syncwarp();  // xs is rewritten for the next sequence
   }
 }
 

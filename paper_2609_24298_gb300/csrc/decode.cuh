@@ -59,95 +59,139 @@ struct Heads {
 };
 
 // ---------------------------------------------------------------------------------------
+// Per-head kernels (query projection, combine): one CTA of 256 threads per (layer, kv head),
+// looping over the sequences 32 query vectors at a time, with the head's basis staged in
+// shared memory once.  The workspace's head-group table gives the group of (head, seq).
+// ---------------------------------------------------------------------------------------
+constexpr int kHeadThreads = 256;
+constexpr int kVecPass = 32;  // query vectors (sequences x G) per pass
+constexpr int kWLd = 132;     // padded row stride (floats) of a staged basis: conflict-free row reads
+constexpr int kZLd = 36;      // row stride of the transposed rank-space averages
+
+__host__ __device__ constexpr size_t qproj_smem_bytes() {
+  return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd);
+}
+__host__ __device__ constexpr size_t combine_smem_bytes() {
+  return sizeof(float) * ((size_t)kD * kD + (size_t)kD * kZLd + kD);
+}
+
+// ---------------------------------------------------------------------------------------
 // a4: query projection
+//   q~_g = (Delta_K / sqrt d) log2(e) W_K^T q_g per query head, scaled by a power of two so
+//   that max |q~| of the group lands in [256, 512), split into fp16 hi + lo and laid out as
+//   the scan's MMA B fragments; Qsum_g = sum over channels of the fed hi + lo values.
 // ---------------------------------------------------------------------------------------
 template <int G>
-__global__ void __launch_bounds__(128) qproj_kernel(DecodeArgs a) {
-  constexpr int NTK = Heads<G>::NTK;
+__global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
+  constexpr int NTK = Heads<G>::NTK, SPP = kVecPass / G;
+  extern __shared__ __align__(16) float qsm[];
+  float* Ws = qsm;                  // [kD][kWLd]   W_K row i = channel i
+  float* Qs = Ws + kD * kWLd;       // [kVecPass][kD] queries of this pass (fp32)
+  float* Os = Qs + kVecPass * kD;   // [kVecPass][kWLd] scaled q~ of this pass
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
-  const WsGroup gr = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off)[blockIdx.x];
-  const HeadEntry hk = head_table(a.block)[gr.k_head];
+  const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
+  const int S = wh->n_seqs;
+  const int* hg = reinterpret_cast<const int*>(a.ws + wh->hg_off) + (size_t)blockIdx.x * S;
+  const WsGroup g0 = groups[hg[0]];
+  const HeadEntry hk = head_table(a.block)[g0.k_head];
   const float* pool = param_pool(a.block);
-  unsigned char* qt = a.ws + wh->qt_off + (size_t)blockIdx.x * wh->qt_stride;
-  const int r = hk.r;
-  __shared__ float qs[G][kD];
-  __shared__ float qv[G][kD];
-  __shared__ float red[4];
-  const int tid = threadIdx.x;
-  const __nv_bfloat16* qp = a.q + gr.layer * a.q_sl + gr.seq * a.q_ss + (long long)gr.kv * G * kD;
-#pragma unroll
-  for (int g = 0; g < G; ++g) qv[g][tid] = __bfloat162float(qp[g * kD + tid]);
-  __syncthreads();
-  // q~[g][i] for channel i = tid
+  const int r = hk.r, layer = g0.layer, kv = g0.kv;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float scale = hk.delta * 0.088388347648318440f * 1.4426950408889634f;  // Delta/sqrt(128)*log2(e)
-  float vals[G];
-  float amax = 0.f;
-#pragma unroll
-  for (int g = 0; g < G; ++g) vals[g] = 0.f;
-  if (tid < r) {
-    const float* w = pool + hk.w_off + (size_t)tid * kD;
-    for (int dd = 0; dd < kD; dd += 4) {
-      const float4 wv = *reinterpret_cast<const float4*>(w + dd);
-#pragma unroll
-      for (int g = 0; g < G; ++g)
-        vals[g] += wv.x * qv[g][dd] + wv.y * qv[g][dd + 1] + wv.z * qv[g][dd + 2] + wv.w * qv[g][dd + 3];
+  stage_basis(pool + hk.w_off, r, kWLd, Ws);
+  for (int s0 = 0; s0 < S; s0 += SPP) {
+    const int ns = min(SPP, S - s0), nv = ns * G;
+    __syncthreads();  // basis staged; the previous pass is done with Qs and Os
+    // queries are only 2-byte aligned in general: element loads, all issued together
+#pragma unroll 16
+    for (int idx = tid; idx < nv * kD; idx += kHeadThreads) {
+      const int v = idx / kD, d = idx % kD;
+      const __nv_bfloat16* qp = a.q + layer * a.q_sl + (long long)(s0 + v / G) * a.q_ss + (long long)(kv * G + v % G) * kD;
+      Qs[v * kD + d] = __bfloat162float(qp[d]);
     }
+    __syncthreads();
+    // warp w: vectors 4w..4w+3; lane: channels lane + 32c
+    const int v0 = 4 * warp;
+    if (v0 < nv) {
+      float acc[4][4];
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      vals[g] *= scale;
-      amax = fmaxf(amax, fabsf(vals[g]));
-    }
-  }
-  // power-of-two scale so that max |q~| lands in [256, 512)
+      for (int c = 0; c < 4; ++c)
 #pragma unroll
-  for (int o = 16; o; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-  if ((tid & 31) == 0) red[tid >> 5] = amax;
-  __syncthreads();
-  amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-  int e = 0;
-  if (amax > 0.f) {
-    int ex;
-    frexpf(amax, &ex);  // amax = m 2^ex, m in [0.5, 1)
-    e = 9 - ex;
-  }
-  const float up = ldexpf(1.f, e);
+        for (int v = 0; v < 4; ++v) acc[c][v] = 0.f;
+#pragma unroll 4
+      for (int d = 0; d < kD; d += 4) {
+        float4 w[4], q[4];
 #pragma unroll
-  for (int g = 0; g < G; ++g) qs[g][tid] = vals[g] * up;
-  __syncthreads();
-  // sums of the fp16 hi+lo values actually fed to the MMA (scaled units)
-  float* qhdr = reinterpret_cast<float*>(qt);
-  if (tid < G) {
-    float s = 0.f;
-    for (int i = 0; i < r; ++i) {
-      const float x = qs[tid][i];
-      const __half h = __float2half_rn(x);
-      const __half l = __float2half_rn(x - __half2float(h));
-      s += __half2float(h) + __half2float(l);
-    }
-    qhdr[tid] = s;
-  }
-  if (tid == 0) qhdr[8] = ldexpf(1.f, -e);
-  // B fragments [kappa][nt][lane] uint2: element (k, n) = hi or lo part of q~ of channel
-  // 16 kappa + k for the query head of column n (see Heads)
-  uint2* frag = reinterpret_cast<uint2*>(qt + kQtHeaderBytes);
-  for (int idx = tid; idx < 8 * NTK * 32; idx += 128) {
-    const int lane = idx & 31, nt = (idx >> 5) % NTK, kap = idx / (32 * NTK);
-    const int j = lane & 3, n = lane >> 2;
-    const int g = Heads<G>::col_head(nt, n), lo = Heads<G>::col_lo(nt, n);
-    float e4[4];
-    const int ks[4] = {2 * j, 2 * j + 1, 2 * j + 8, 2 * j + 9};
+        for (int c = 0; c < 4; ++c) w[c] = *reinterpret_cast<const float4*>(Ws + (lane + 32 * c) * kWLd + d);
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int ch = 16 * kap + ks[u];
-      float v = 0.f;
-      if (ch < r) {
-        const float x = qs[g][ch];
-        const float h = __half2float(__float2half_rn(x));
-        v = lo ? (x - h) : h;
+        for (int v = 0; v < 4; ++v) q[v] = *reinterpret_cast<const float4*>(Qs + (v0 + v) * kD + d);
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            acc[c][v] += w[c].x * q[v].x + w[c].y * q[v].y + w[c].z * q[v].z + w[c].w * q[v].w;
       }
-      e4[u] = v;
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) Os[(v0 + v) * kWLd + lane + 32 * c] = acc[c][v] * scale;
     }
-    frag[(kap * 2 + nt) * 32 + lane] = make_uint2(pack_f16(e4[0], e4[1]), pack_f16(e4[2], e4[3]));
+    __syncthreads();
+    // per sequence (one warp each): power-of-two scale, hi/lo split, Qsum, B fragments
+    for (int sl = warp; sl < ns; sl += kHeadThreads / 32) {
+      const float* o = Os + sl * G * kWLd;
+      float amax = 0.f;
+      for (int i = lane; i < r; i += 32)
+#pragma unroll
+        for (int g = 0; g < G; ++g) amax = fmaxf(amax, fabsf(o[g * kWLd + i]));
+#pragma unroll
+      for (int m = 16; m; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, m));
+      int e = 0;
+      if (amax > 0.f) {
+        int ex;
+        frexpf(amax, &ex);  // amax = m 2^ex, m in [0.5, 1)
+        e = 9 - ex;
+      }
+      const float up = ldexpf(1.f, e);
+      unsigned char* qt = a.ws + wh->qt_off + (size_t)hg[s0 + sl] * wh->qt_stride;
+      float* qhdr = reinterpret_cast<float*>(qt);
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        float sum = 0.f;
+        for (int i = lane; i < r; i += 32) {
+          const float x = o[g * kWLd + i] * up;
+          const __half h = __float2half_rn(x);
+          const __half l = __float2half_rn(x - __half2float(h));
+          sum += __half2float(h) + __half2float(l);
+        }
+#pragma unroll
+        for (int m = 16; m; m >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, m);
+        if (lane == 0) qhdr[g] = sum;
+      }
+      if (lane == 0) qhdr[8] = ldexpf(1.f, -e);
+      // element (k, n) of fragment (kappa, nt) = hi or lo part of q~ of channel 16 kappa + k
+      // for the query head of column n (see Heads)
+      uint2* frag = reinterpret_cast<uint2*>(qt + kQtHeaderBytes);
+      for (int idx = lane; idx < 8 * NTK * 32; idx += 32) {
+        const int fl = idx & 31, nt = (idx >> 5) % NTK, kap = idx / (32 * NTK);
+        const int j = fl & 3, n = fl >> 2;
+        const int g = Heads<G>::col_head(nt, n), lo = Heads<G>::col_lo(nt, n);
+        float e4[4];
+        const int ks[4] = {2 * j, 2 * j + 1, 2 * j + 8, 2 * j + 9};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int ch = 16 * kap + ks[u];
+          float v = 0.f;
+          if (ch < r) {
+            const float x = o[g * kWLd + ch] * up;
+            const float h = __half2float(__float2half_rn(x));
+            v = lo ? (x - h) : h;
+          }
+          e4[u] = v;
+        }
+        frag[(kap * 2 + nt) * 32 + fl] = make_uint2(pack_f16(e4[0], e4[1]), pack_f16(e4[2], e4[3]));
+      }
+    }
   }
 }
 
@@ -617,52 +661,139 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
 
 // ---------------------------------------------------------------------------------------
 // a7: combine chunks + back-projection
+//   per query head: m* = max over chunks, l* = sum 2^(m - m*) l, zbar = Delta_V (sum 2^(m - m*)
+//   acc / l* - 2^{b-1} + 1/2), o = mu_V + W_V zbar (zeros for an empty sequence).
 // ---------------------------------------------------------------------------------------
 template <int G>
-__global__ void __launch_bounds__(128) combine_kernel(DecodeArgs a) {
+__global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
+  constexpr int SPP = kVecPass / G;
+  extern __shared__ __align__(16) float csm[];
+  float* Ws = csm;                  // [kD][kD]     W_V row i = channel i
+  float* Zs = Ws + kD * kD;         // [kD][kZLd]   zbar of this pass, [channel][vector]
+  float* mus = Zs + kD * kZLd;      // [kD]         mu_V
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
-  const WsGroup gr = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off)[blockIdx.x];
-  const HeadEntry hv = head_table(a.block)[gr.v_head];
-  const float* pool = param_pool(a.block);
+  const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
   const float* parts = reinterpret_cast<const float*>(a.ws + wh->part_off);
+  const int S = wh->n_seqs;
+  const int* hg = reinterpret_cast<const int*>(a.ws + wh->hg_off) + (size_t)blockIdx.x * S;
+  const WsGroup g0 = groups[hg[0]];
+  const HeadEntry hv = head_table(a.block)[g0.v_head];
+  const float* pool = param_pool(a.block);
+  const int rv = hv.r, layer = g0.layer, kv = g0.kv;
   const int tid = threadIdx.x;
-  float* out = a.out + gr.layer * a.o_sl + gr.seq * a.o_ss + (long long)gr.kv * G * kD;
-  const int T = a.seq_lens[gr.seq];
-  if (T <= 0) {
+  const float cen = rv > 0 ? (float)(1 << (hv.b - 1)) - 0.5f : 0.f;
+  stage_basis(pool + hv.w_off, rv, kD, Ws);
+  if (tid < kD) mus[tid] = pool[hv.mu_off + tid];
+  for (int s0 = 0; s0 < S; s0 += SPP) {
+    const int ns = min(SPP, S - s0), nv = ns * G;
+    __syncthreads();  // basis staged; the previous pass is done with Zs
+    // warp w: vectors w, w + 8, w + 16, w + 24 together (their partial loads overlap);
+    // lane: channels lane + 32c
+    {
+      const int warp = tid >> 5, lane = tid & 31;
+      constexpr int NU = kVecPass / (kHeadThreads / 32);
+      const float* pg0[NU];
+      int ni[NU], gi[NU];
+      bool live[NU];
+      float mst[NU], lst[NU], acc[NU][4];
+      int kmax = 0;
 #pragma unroll
-    for (int g = 0; g < G; ++g) out[g * kD + tid] = 0.f;
-    return;
-  }
-  __shared__ float zbar[G][kD];
-  __shared__ float wts[G][64];
-  const int rv = hv.r, ni = gr.n_items;
-  const float cen = hv.r > 0 ? (float)(1 << (hv.b - 1)) - 0.5f : 0.f;
-  for (int g = 0; g < G; ++g) {
-    float mstar = -INFINITY;
-    for (int k = 0; k < ni; ++k) mstar = fmaxf(mstar, parts[(size_t)(gr.first_item + k) * wh->part_stride + g * wh->g_stride]);
-    float lstar = 0.f, acc = 0.f;
-    for (int k = 0; k < ni; ++k) {
-      const float* pg = parts + (size_t)(gr.first_item + k) * wh->part_stride + g * wh->g_stride;
-      const float w = (pg[0] == -INFINITY) ? 0.f : exp2f(pg[0] - mstar);
-      lstar += w * pg[1];
-      if (tid < rv && w != 0.f) acc += w * pg[4 + tid];
+      for (int u = 0; u < NU; ++u) {
+        const int v = warp + 8 * u;
+        live[u] = v < nv;
+        const WsGroup gr = groups[hg[s0 + (live[u] ? v : 0) / G]];
+        live[u] = live[u] && a.seq_lens[gr.seq] > 0;
+        gi[u] = v % G;
+        ni[u] = live[u] ? gr.n_items : 0;
+        pg0[u] = parts + (size_t)gr.first_item * wh->part_stride + gi[u] * wh->g_stride;
+        kmax = max(kmax, ni[u]);
+        lst[u] = 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[u][c] = 0.f;
+      }
+      // running maxima over the chunks: the loads of all four vectors are issued together
+      {
+        float m[NU];
+#pragma unroll
+        for (int u = 0; u < NU; ++u) m[u] = -INFINITY;
+        for (int k = lane; k < kmax; k += 32)
+#pragma unroll
+          for (int u = 0; u < NU; ++u)
+            m[u] = fmaxf(m[u], k < ni[u] ? pg0[u][(size_t)k * wh->part_stride] : -INFINITY);
+#pragma unroll
+        for (int u = 0; u < NU; ++u) {
+#pragma unroll
+          for (int o = 16; o; o >>= 1) m[u] = fmaxf(m[u], __shfl_xor_sync(0xffffffffu, m[u], o));
+          mst[u] = m[u];
+        }
+      }
+      // weighted sums: every load of a chunk is issued before any weight is applied (a chunk
+      // with no tokens has m = -inf and no value entries, so its weight selects zero)
+      const int nch = min(4, (rv + 31) >> 5);
+#pragma unroll 2
+      for (int k = 0; k < kmax; ++k) {
+        float mk[NU], lk[NU], xk[NU][4];
+#pragma unroll
+        for (int u = 0; u < NU; ++u) {
+          const float* pg = pg0[u] + (size_t)min(k, max(ni[u] - 1, 0)) * wh->part_stride;
+          mk[u] = pg[0];
+          lk[u] = pg[1];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) xk[u][c] = c < nch ? pg[4 + min(lane + 32 * c, rv - 1)] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < NU; ++u) {
+          const bool use = k < ni[u] && mk[u] != -INFINITY;
+          const float w = use ? exp2f(mk[u] - mst[u]) : 0.f;
+          lst[u] += use ? w * lk[u] : 0.f;
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[u][c] += use ? w * xk[u][c] : 0.f;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < NU; ++u) {
+        const int v = warp + 8 * u;
+        if (v >= nv) continue;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int i = lane + 32 * c;
+          Zs[i * kZLd + v] = (live[u] && i < rv) ? hv.delta * (acc[u][c] / lst[u] - cen) : 0.f;
+        }
+      }
     }
-    if (tid < rv) zbar[g][tid] = hv.delta * (acc / lstar - cen);
+    __syncthreads();
+    // thread: dims 4 (tid % 32) .. +3 for vectors 4 (tid / 32) .. +3
+    const int d0 = 4 * (tid & 31), v0 = 4 * (tid >> 5);
+    if (v0 < nv) {
+      const float4 m4 = *reinterpret_cast<const float4*>(mus + d0);
+      float4 o[4] = {m4, m4, m4, m4};
+      for (int i = 0; i < rv; ++i) {
+        const float4 w = *reinterpret_cast<const float4*>(Ws + i * kD + d0);
+        const float4 z = *reinterpret_cast<const float4*>(Zs + i * kZLd + v0);
+        const float zz[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          o[v].x += w.x * zz[v];
+          o[v].y += w.y * zz[v];
+          o[v].z += w.z * zz[v];
+          o[v].w += w.w * zz[v];
+        }
+      }
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int vv = v0 + v;
+        if (vv >= nv) break;
+        const int seq = s0 + vv / G, g = vv % G;
+        const bool empty = a.seq_lens[groups[hg[seq]].seq] <= 0;
+        float* out = a.out + layer * a.o_sl + seq * a.o_ss + (long long)(kv * G + g) * kD + d0;
+        const float4 y = empty ? make_float4(0.f, 0.f, 0.f, 0.f) : o[v];
+        out[0] = y.x;  // the output is only 4-byte aligned in general
+        out[1] = y.y;
+        out[2] = y.z;
+        out[3] = y.w;
+      }
+    }
   }
-  (void)wts;
-  __syncthreads();
-  const float* W = pool + hv.w_off;
-  const float mu = pool[hv.mu_off + tid];
-  float o[G];
-#pragma unroll
-  for (int g = 0; g < G; ++g) o[g] = mu;
-  for (int i = 0; i < rv; ++i) {
-    const float w = W[(size_t)i * kD + tid];
-#pragma unroll
-    for (int g = 0; g < G; ++g) o[g] += w * zbar[g][i];
-  }
-#pragma unroll
-  for (int g = 0; g < G; ++g) out[g * kD + tid] = o[g];
 }
 
 }  // namespace cobra

@@ -763,6 +763,8 @@ void ws_layout(const cobra_decode_desc* d, const Plan& p, cobra::WsHeader& h, si
   off += sizeof(cobra::WsGroup) * p.groups.size();
   h.items_off = off = align_up(off, 256);
   off += sizeof(cobra::WsItem) * p.items.size();
+  h.hg_off = off = align_up(off, 256);
+  off += sizeof(int32_t) * p.groups.size();
   h.qt_off = off = align_up(off, 256);
   off += (size_t)h.qt_stride * p.groups.size();
   h.part_off = off = align_up(off, 256);
@@ -794,11 +796,16 @@ extern "C" cobra_status cobra_decode_plan(const cobra_decode_desc* desc, const i
   size_t need;
   ws_layout(desc, p, h, need);
   if (ws_bytes < need) return COBRA_ESPACE;
-  const size_t head_bytes = h.qt_off;  // header + groups + items
+  const size_t head_bytes = h.qt_off;  // header + groups + items + head-group table
   std::vector<unsigned char> img(head_bytes, 0);
   std::memcpy(img.data(), &h, sizeof(h));
   std::memcpy(img.data() + h.groups_off, p.groups.data(), sizeof(cobra::WsGroup) * p.groups.size());
   std::memcpy(img.data() + h.items_off, p.items.data(), sizeof(cobra::WsItem) * p.items.size());
+  int32_t* hg = reinterpret_cast<int32_t*>(img.data() + h.hg_off);
+  for (size_t g = 0; g < p.groups.size(); ++g) {
+    const cobra::WsGroup& gr = p.groups[g];
+    hg[((size_t)gr.layer * desc->n_kv_heads + gr.kv) * desc->n_seqs + gr.seq] = (int32_t)g;
+  }
   cudaStream_t s = (cudaStream_t)stream;
   if (cudaMemcpyAsync(workspace, img.data(), head_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess) return COBRA_ECUDA;
   if (cudaStreamSynchronize(s) != cudaSuccess) return COBRA_ECUDA;

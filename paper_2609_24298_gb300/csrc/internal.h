@@ -36,7 +36,7 @@ struct HeadEntry {
 };
 static_assert(sizeof(HeadEntry) == 64, "head entry size");
 
-// Decode workspace: header | groups | items | q~ blocks | partials.
+// Decode workspace: header | groups | items | head-group table | q~ blocks | partials.
 struct WsHeader {
   uint32_t magic;
   uint32_t version;
@@ -52,7 +52,9 @@ struct WsHeader {
   int32_t qt_stride;    // bytes per group q~ block
   int32_t max_rv;
   int32_t max_row_bytes;  // largest K or V code row among the planned heads
-  int32_t reserved[11];
+  int32_t reserved0;
+  uint64_t hg_off;        // int32 [n_layers * n_kv][n_seqs]: group index of (head, seq)
+  int32_t reserved[8];
 };
 static_assert(sizeof(WsHeader) == 128, "ws header size");
 

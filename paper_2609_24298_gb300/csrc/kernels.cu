@@ -191,10 +191,16 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
   a.n_seqs = d->n_seqs;
   a.rows_per_seq = d->rows_per_seq;
   a.pages_per_seq = d->pages_per_seq;
-  const long long warps = (long long)d->n_layers * d->n_kv_heads * d->n_seqs;
-  const long long grid = (warps + 3) / 4;
+  const long long grid = (long long)d->n_layers * d->n_kv_heads;  // one CTA per (layer, kv head)
   if (grid > 0x7fffffffLL) return COBRA_EINVAL;
-  append_kernel<<<(unsigned)grid, 128, 0, (cudaStream_t)stream>>>(a);
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_smem_bytes()) !=
+        cudaSuccess)
+      return COBRA_ECUDA;
+    attr = true;
+  }
+  append_kernel<<<(unsigned)grid, kAppendThreads, append_smem_bytes(), (cudaStream_t)stream>>>(a);
   return launch_status();
 }
 
@@ -204,9 +210,18 @@ size_t decode_osm_bytes_host(int G) { return (size_t)8 * 32 * (G == 4 ? 2 : 4) *
 enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
 template <int G>
-cobra_status launch_decode(const DecodeArgs& a, int n_groups, int n_items, int stages, cudaStream_t s) {
+cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_items, int stages, cudaStream_t s) {
+  static bool head_attr = false;
+  if (!head_attr) {
+    if (cudaFuncSetAttribute(qproj_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)qproj_smem_bytes()) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(combine_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)combine_smem_bytes()) != cudaSuccess)
+      return COBRA_ECUDA;
+    head_attr = true;
+  }
   if (stages & kQproj) {
-    qproj_kernel<G><<<n_groups, 128, 0, s>>>(a);
+    qproj_kernel<G><<<n_heads, kHeadThreads, qproj_smem_bytes(), s>>>(a);
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kScan) {
@@ -227,7 +242,7 @@ cobra_status launch_decode(const DecodeArgs& a, int n_groups, int n_items, int s
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kCombine) {
-    combine_kernel<G><<<n_groups, 128, 0, s>>>(a);
+    combine_kernel<G><<<n_heads, kHeadThreads, combine_smem_bytes(), s>>>(a);
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   return COBRA_OK;
@@ -267,8 +282,10 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   // 8 KB of row staging per warp, or two of the largest rows if those are bigger
   a.ring_bytes = (int)std::max<size_t>(8192, 2 * align_up((size_t)rowb, 128));
   cudaStream_t s = (cudaStream_t)stream;
-  if (d->group == 4) return launch_decode<4>(a, info->n_groups, info->n_items, stages, s);
-  return launch_decode<8>(a, info->n_groups, info->n_items, stages, s);
+  const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
+  if (n_heads * d->n_seqs != info->n_groups) return COBRA_EINVAL;  // plan made for another descriptor
+  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, info->n_items, stages, s);
+  return launch_decode<8>(a, (int)n_heads, info->n_items, stages, s);
 }
 }  // namespace
 
@@ -335,7 +352,7 @@ cobra_status static_scratch(unsigned char** out) {
 
 // Workspace layout for a one-chunk-per-group plan with room for any head (r_V <= 128).
 struct StaticPlanSizes {
-  size_t groups_off, items_off, qt_off, part_off, total;
+  size_t groups_off, items_off, hg_off, qt_off, part_off, total;
   int g_stride, part_stride;
 };
 StaticPlanSizes static_plan_sizes(int n_groups, int group) {
@@ -347,6 +364,8 @@ StaticPlanSizes static_plan_sizes(int n_groups, int group) {
   off = align_up(off + sizeof(WsGroup) * (size_t)n_groups, 256);
   z.items_off = off;
   off = align_up(off + sizeof(WsItem) * (size_t)n_groups, 256);
+  z.hg_off = off;
+  off = align_up(off + sizeof(int) * (size_t)n_groups, 256);
   z.qt_off = off;
   off = align_up(off + (size_t)kQtStride * n_groups, 256);
   z.part_off = off;
@@ -362,12 +381,14 @@ __global__ void static_plan_kernel(unsigned char* ws, const unsigned char* block
                                    StaticPlanSizes z, int n_groups, int cap_rows) {
   WsGroup* groups = reinterpret_cast<WsGroup*>(ws + z.groups_off);
   WsItem* items = reinterpret_cast<WsItem*>(ws + z.items_off);
+  int* hg = reinterpret_cast<int*>(ws + z.hg_off);
   const HeadEntry* heads = head_table(block);
   for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < n_groups; g += gridDim.x * blockDim.x) {
     const int h = g % d.n_kv_heads, l = (g / d.n_kv_heads) % d.n_layers, s = g / (d.n_kv_heads * d.n_layers);
     const int hk = d.k_head0 + l * d.layer_stride + h, hv = d.v_head0 + l * d.layer_stride + h;
     groups[g] = WsGroup{s, l, h, g, 1, hk, hv, 0};
     items[g] = WsItem{g, 0, cap_rows, 0};
+    hg[((size_t)l * d.n_kv_heads + h) * d.n_seqs + s] = g;
     (void)heads;
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -383,6 +404,7 @@ __global__ void static_plan_kernel(unsigned char* ws, const unsigned char* block
     hd.n_seqs = d.n_seqs;
     hd.groups_off = z.groups_off;
     hd.items_off = z.items_off;
+    hd.hg_off = z.hg_off;
     hd.qt_off = z.qt_off;
     hd.part_off = z.part_off;
     hd.part_stride = z.part_stride;
@@ -434,8 +456,9 @@ extern "C" cobra_status cobra_decode_attn_static(const void* params, const cobra
   a.pages_per_seq = d->pages_per_seq;
   a.one = kOneH2;
   a.ring_bytes = 2 * 16 * kD * 8;  // two rows of the largest head (r = 128, b = 8)
-  if (d->group == 4) return launch_decode<4>(a, (int)n_groups, (int)n_groups, kQproj | kScan | kCombine, s);
-  return launch_decode<8>(a, (int)n_groups, (int)n_groups, kQproj | kScan | kCombine, s);
+  const int n_heads = d->n_layers * d->n_kv_heads;
+  if (d->group == 4) return launch_decode<4>(a, n_heads, (int)n_groups, kQproj | kScan | kCombine, s);
+  return launch_decode<8>(a, n_heads, (int)n_groups, kQproj | kScan | kCombine, s);
 }
 
 extern "C" cobra_status cobra_check(void* stream) {
