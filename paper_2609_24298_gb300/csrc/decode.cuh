@@ -71,8 +71,9 @@ constexpr int kZLd = 36;      // row stride of the transposed rank-space average
 __host__ __device__ constexpr size_t qproj_smem_bytes() {
   return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd);
 }
+constexpr int kWtChunk = 64;  // chunk weights held in shared memory per vector and round
 __host__ __device__ constexpr size_t combine_smem_bytes() {
-  return sizeof(float) * ((size_t)kD * kD + (size_t)kD * kZLd + kD);
+  return sizeof(float) * ((size_t)kD * kD + (size_t)kD * kZLd + kD + (size_t)kVecPass * kWtChunk);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -467,7 +468,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
   int outstanding = 0;      // loads issued but not yet waited for
   int wait_stage = 0, nstage = 2;
 
-  for (int item = blockIdx.x * kDecodeWarps + warp; item < n_items && !failed; item += gridDim.x * kDecodeWarps) {
+  // work items are taken in plan order from a shared counter, so that warps that finish early
+  // take more (the items' costs differ with the heads' bit widths)
+  unsigned int* next_item = const_cast<unsigned int*>(&wh->next_item);
+  auto take = [&]() -> int {
+    int v = 0;
+    if (lane == 0) v = (int)atomicAdd(next_item, 1u);
+    return __shfl_sync(0xffffffffu, v, 0);
+  };
+  for (int item = take(); item < n_items && !failed; item = take()) {
     const WsItem it = items[item];
     const WsGroup gr = groups[it.group];
     const int kr = heads[gr.k_head].r, kb = heads[gr.k_head].b, vr = heads[gr.v_head].r, vb = heads[gr.v_head].b;
@@ -671,6 +680,9 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   float* Ws = csm;                  // [kD][kD]     W_V row i = channel i
   float* Zs = Ws + kD * kD;         // [kD][kZLd]   zbar of this pass, [channel][vector]
   float* mus = Zs + kD * kZLd;      // [kD]         mu_V
+  float* wts = mus + kD;            // [kVecPass][kWtChunk] normalised chunk weights
+  __shared__ float vinfo_m[kVecPass], vinfo_inv_l[kVecPass];
+  __shared__ int vinfo_first[kVecPass], vinfo_n[kVecPass], vinfo_g[kVecPass];
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
   const float* parts = reinterpret_cast<const float*>(a.ws + wh->part_off);
@@ -687,78 +699,125 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   for (int s0 = 0; s0 < S; s0 += SPP) {
     const int ns = min(SPP, S - s0), nv = ns * G;
     __syncthreads();  // basis staged; the previous pass is done with Zs
-    // warp w: vectors w, w + 8, w + 16, w + 24 together (their partial loads overlap);
-    // lane: channels lane + 32c
+    // (1) per vector (warp w: vectors w, w + 8, w + 16, w + 24): m* = max over the chunks and
+    //     l* = sum 2^(m - m*) l, lanes over chunks, merged online (a chunk with no tokens has
+    //     m = -inf and no value entries; its weight is zero).  The four vectors' loads are
+    //     issued together.
+    const int warp = tid >> 5, lane = tid & 31;
+    constexpr int NU = kVecPass / (kHeadThreads / 32);
     {
-      const int warp = tid >> 5, lane = tid & 31;
-      constexpr int NU = kVecPass / (kHeadThreads / 32);
       const float* pg0[NU];
-      int ni[NU], gi[NU];
-      bool live[NU];
-      float mst[NU], lst[NU], acc[NU][4];
+      int ni[NU];
+      float M[NU], Lsum[NU];
       int kmax = 0;
 #pragma unroll
       for (int u = 0; u < NU; ++u) {
         const int v = warp + 8 * u;
-        live[u] = v < nv;
-        const WsGroup gr = groups[hg[s0 + (live[u] ? v : 0) / G]];
-        live[u] = live[u] && a.seq_lens[gr.seq] > 0;
-        gi[u] = v % G;
-        ni[u] = live[u] ? gr.n_items : 0;
-        pg0[u] = parts + (size_t)gr.first_item * wh->part_stride + gi[u] * wh->g_stride;
+        const WsGroup gr = groups[hg[s0 + min(v, nv - 1) / G]];
+        ni[u] = (v < nv && a.seq_lens[gr.seq] > 0) ? gr.n_items : 0;
+        pg0[u] = parts + (size_t)gr.first_item * wh->part_stride + (v % G) * wh->g_stride;
+        M[u] = -INFINITY;
+        Lsum[u] = 0.f;
         kmax = max(kmax, ni[u]);
-        lst[u] = 0.f;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) acc[u][c] = 0.f;
-      }
-      // running maxima over the chunks: the loads of all four vectors are issued together
-      {
-        float m[NU];
-#pragma unroll
-        for (int u = 0; u < NU; ++u) m[u] = -INFINITY;
-        for (int k = lane; k < kmax; k += 32)
-#pragma unroll
-          for (int u = 0; u < NU; ++u)
-            m[u] = fmaxf(m[u], k < ni[u] ? pg0[u][(size_t)k * wh->part_stride] : -INFINITY);
-#pragma unroll
-        for (int u = 0; u < NU; ++u) {
-#pragma unroll
-          for (int o = 16; o; o >>= 1) m[u] = fmaxf(m[u], __shfl_xor_sync(0xffffffffu, m[u], o));
-          mst[u] = m[u];
+        if (v < nv && lane == 0) {
+          vinfo_first[v] = ni[u] > 0 ? gr.first_item : -1;
+          vinfo_n[v] = ni[u];
+          vinfo_g[v] = v % G;
         }
       }
-      // weighted sums: every load of a chunk is issued before any weight is applied (a chunk
-      // with no tokens has m = -inf and no value entries, so its weight selects zero)
-      const int nch = min(4, (rv + 31) >> 5);
-#pragma unroll 2
-      for (int k = 0; k < kmax; ++k) {
-        float mk[NU], lk[NU], xk[NU][4];
+      for (int k = lane; k < kmax; k += 32) {
+        float mk[NU], lk[NU];
 #pragma unroll
         for (int u = 0; u < NU; ++u) {
-          const float* pg = pg0[u] + (size_t)min(k, max(ni[u] - 1, 0)) * wh->part_stride;
-          mk[u] = pg[0];
-          lk[u] = pg[1];
-#pragma unroll
-          for (int c = 0; c < 4; ++c) xk[u][c] = c < nch ? pg[4 + min(lane + 32 * c, rv - 1)] : 0.f;
+          const bool ok = k < ni[u];
+          mk[u] = ok ? pg0[u][(size_t)k * wh->part_stride] : -INFINITY;
+          lk[u] = ok ? pg0[u][(size_t)k * wh->part_stride + 1] : 0.f;
         }
 #pragma unroll
         for (int u = 0; u < NU; ++u) {
-          const bool use = k < ni[u] && mk[u] != -INFINITY;
-          const float w = use ? exp2f(mk[u] - mst[u]) : 0.f;
-          lst[u] += use ? w * lk[u] : 0.f;
-#pragma unroll
-          for (int c = 0; c < 4; ++c) acc[u][c] += use ? w * xk[u][c] : 0.f;
+          if (mk[u] == -INFINITY) continue;
+          const float mn = fmaxf(M[u], mk[u]);
+          Lsum[u] = Lsum[u] * exp2f(M[u] - mn) + lk[u] * exp2f(mk[u] - mn);
+          M[u] = mn;
         }
       }
 #pragma unroll
       for (int u = 0; u < NU; ++u) {
-        const int v = warp + 8 * u;
-        if (v >= nv) continue;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const int i = lane + 32 * c;
-          Zs[i * kZLd + v] = (live[u] && i < rv) ? hv.delta * (acc[u][c] / lst[u] - cen) : 0.f;
+        for (int o = 16; o; o >>= 1) {
+          const float mo = __shfl_xor_sync(0xffffffffu, M[u], o), lo = __shfl_xor_sync(0xffffffffu, Lsum[u], o);
+          const float mn = fmaxf(M[u], mo);
+          if (mn != -INFINITY) {
+            Lsum[u] = Lsum[u] * exp2f(M[u] - mn) + lo * exp2f(mo - mn);
+            M[u] = mn;
+          }
         }
+        const int v = warp + 8 * u;
+        if (v < nv && lane == 0) {
+          vinfo_m[v] = M[u];
+          vinfo_inv_l[v] = ni[u] > 0 ? 1.f / Lsum[u] : 0.f;
+        }
+      }
+    }
+    __syncthreads();
+    // (2) zbar[v][i] = Delta (sum_k w_k acc_k[i] - 2^{b-1} + 1/2) with w_k = 2^(m_k - m*) / l*.
+    //     Rounds of kWtChunk chunks: the weights of a round are computed one (vector, chunk) per
+    //     thread into shared memory; then thread (channel i, vector parity) sums over them in
+    //     blocks of 4 vectors x 8 chunks whose 32 loads are all issued before any is used.
+    {
+      const int i = tid & (kD - 1), par = tid >> 7;
+      int kmax = 0;
+      for (int v = 0; v < nv; ++v) kmax = max(kmax, vinfo_n[v]);
+      float acc[kVecPass / 2];
+#pragma unroll
+      for (int q = 0; q < kVecPass / 2; ++q) acc[q] = 0.f;
+      for (int k0 = 0; k0 < kmax; k0 += kWtChunk) {
+        __syncthreads();  // the previous round's weights are consumed
+        for (int idx = tid; idx < nv * kWtChunk; idx += kHeadThreads) {
+          const int v = idx / kWtChunk, k = k0 + idx % kWtChunk;
+          float w = 0.f;
+          if (k < vinfo_n[v]) {
+            const float mk = parts[(size_t)(vinfo_first[v] + k) * wh->part_stride + vinfo_g[v] * wh->g_stride];
+            if (mk != -INFINITY) w = exp2f(mk - vinfo_m[v]) * vinfo_inv_l[v];
+          }
+          wts[idx] = w;
+        }
+        __syncthreads();
+        if (i >= rv) continue;
+        const int kr = min(kWtChunk, kmax - k0);
+#pragma unroll
+        for (int q0 = 0; q0 < kVecPass / 2; q0 += 4) {
+          if (2 * q0 + par >= nv) break;
+          for (int kb = 0; kb < kr; kb += 8) {
+            float x[4][8];
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+              const int v = 2 * (q0 + qq) + par;
+              const int n = v < nv ? vinfo_n[v] - k0 : 0;
+              const float* px = parts + (size_t)max(vinfo_first[v < nv ? v : 0], 0) * wh->part_stride +
+                                (size_t)k0 * wh->part_stride + (v < nv ? vinfo_g[v] : 0) * wh->g_stride + 4 + i;
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk) x[qq][kk] = (kb + kk < n) ? px[(size_t)(kb + kk) * wh->part_stride] : 0.f;
+            }
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+              const int v = 2 * (q0 + qq) + par;
+              if (v >= nv) break;
+              const float* wv = wts + v * kWtChunk + kb;
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk) {
+                const float w = (kb + kk < kWtChunk) ? wv[kk] : 0.f;
+                acc[q0 + qq] += w != 0.f ? w * x[qq][kk] : 0.f;
+              }
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < kVecPass / 2; ++q) {
+        const int v = 2 * q + par;
+        if (v >= nv) break;
+        Zs[i * kZLd + v] = (i < rv && vinfo_first[v] >= 0) ? hv.delta * (acc[q] - cen) : 0.f;
       }
     }
     __syncthreads();

@@ -671,7 +671,7 @@ extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, 
 // that each chunk reads about kItemBytes of packed K+V codes.
 // ----------------------------------------------------------------------------------------
 namespace {
-constexpr long long kItemBytes = 256 * 1024;
+constexpr long long kItemBytes = 64 * 1024;
 
 cobra_status check_decode_desc(const cobra_decode_desc* d) {
   if (!d) return COBRA_EINVAL;

@@ -1,5 +1,6 @@
 // libcobra device entry points: argument checks and launches for compress, append and
 // decode attention, plus the device status check.
+#include <cstddef>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -238,6 +239,8 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_items, int st
     per_sm = std::max(per_sm, 1);
     const int want = (n_items + kDecodeWarps - 1) / kDecodeWarps;
     const int grid = std::max(1, std::min(want, per_sm * sm_count()));
+    if (cudaMemsetAsync(a.ws + offsetof(WsHeader, next_item), 0, sizeof(uint32_t), s) != cudaSuccess)
+      return COBRA_ECUDA;
     decode_kernel<G><<<grid, kDecodeWarps * 32, smem, s>>>(a);
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
