@@ -66,6 +66,26 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+// The same operations executed only where `p` holds: every lane of a warp runs the address
+// arithmetic and one lane issues, without a divergent branch.
+__device__ __forceinline__ void mbar_arrive_expect_tx_if(bool p, uint32_t bar, uint32_t bytes) {
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %2, 0;\n @q mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n}\n" ::"r"(
+          bar),
+      "r"(bytes), "r"((int)p)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_g2s_if(bool p, uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %4, 0;\n"
+      " @q cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n}\n" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar), "r"((int)p)
+      : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem_if(bool p) {
+  asm volatile("{\n .reg .pred q;\n setp.ne.b32 q, %0, 0;\n @q fence.proxy.async.shared::cta;\n}\n" ::"r"((int)p)
+               : "memory");
+}
 
 // ---------------------------------------------------------------------------------------
 // legacy warp-level MMA (operands in registers) and 8x8 transposition

@@ -199,17 +199,22 @@ __global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
 // ---------------------------------------------------------------------------------------
 // a5 + a6: chunked rank-space scan
 //
-// Per warp: running max m, sum l and offset correction c per owned query head in registers;
-// the rank-space value accumulators (the lane's C-fragment entries of O) live in the warp's
-// shared memory and are rescaled only when the running max moves.  Loops over k-tiles (K
-// side) and channel tiles (V side) stay rolled to keep each (b_K, b_V) variant's code small;
-// only the 8 token tiles of a row are unrolled.
+// Per warp and work item (a run of code rows of one (seq, layer, kv head)):
+//  * each stage of the warp's shared-memory ring holds one K row and the V row of the same
+//    tokens, both copied with cp.async.bulk onto one mbarrier; the copies are issued by one
+//    lane under a predicate, so the warp never diverges;
+//  * scores s_t (log2 units) come from the K codes by f16 MMA; probabilities are taken
+//    against a reference max that is raised (and the accumulators rescaled) only when a
+//    row's max exceeds it by more than kTau, so most rows need no rescale;
+//  * the V MMA accumulates O[i] = sum_t f_t A_t[i] over the fed probabilities f_t.  Two
+//    constant rows appended after the last channel give, in the same accumulators, the sum
+//    of the fed values c (row r: A = 1) and the normaliser l (row r + 1: A = 2^(k - kmin),
+//    which undoes each register's window), so both are rescaled with O.
+// Loops over k-tiles (K side) and channel tiles (V side) stay rolled to keep each bit width's
+// code small; the 8 token tiles of a row are unrolled.
 // ---------------------------------------------------------------------------------------
-template <int G>
-struct WarpState {
-  static constexpr int NG = G / 4;
-  float m[NG], l[NG], c[NG];
-};
+constexpr float kTau = 8.f;    // fed probabilities stay below 2^kTau (fp16 range)
+constexpr int kMaxVTiles = 9;  // channel tiles of the V accumulators: 8 + the one holding rows r, r+1
 
 // accumulator floats per (channel tile, lane): the live C-fragment entries of the V MMA
 template <int G>
@@ -265,7 +270,8 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
   if (nk > nfull) tile(true, nfull);
   // acc = Qsum + 2^(k-10) * sum_i q~_i code_i, Qsum = sum of the q~ fed to the MMA.  b >= 3
   // uses one window for every register, so Qsum shifts every token's score alike and softmax
-  // ignores it; b = 1, 2 mix windows, so Qsum is removed before the per-token rescale.
+  // ignores it; b = 1, 2 mix windows, so Qsum is removed before the per-token rescale:
+  // s = acc * sc - Qsum * sc with sc = scale 2^(10-k).
 #pragma unroll
   for (int t = 0; t < 8; ++t) {
     const float sc0 = qscale * Window<B>::inv_scale(2 * t), sc1 = qscale * Window<B>::inv_scale(2 * t + 1);
@@ -276,8 +282,8 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
       const float v0 = G == 4 ? acc[t][0][0] + acc[t][0][1] : acc[t][0][u] + acc[t][NTK - 1][u];
       const float v1 = G == 4 ? acc[t][0][2] + acc[t][0][3] : acc[t][0][2 + u] + acc[t][NTK - 1][2 + u];
       if constexpr (B <= 2) {
-        s[t][u][0] = (v0 - qsum[u]) * sc0;
-        s[t][u][1] = (v1 - qsum[u]) * sc1;
+        s[t][u][0] = fmaf(v0, sc0, -qsum[u] * sc0);
+        s[t][u][1] = fmaf(v1, sc1, -qsum[u] * sc1);
       } else {
         s[t][u][0] = v0 * sc0;
         s[t][u][1] = v1 * sc1;
@@ -286,25 +292,34 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
   }
 }
 
+// f16x2 constant of the normaliser row for register rho: 2^(k(rho) - kmin) in both halves
+template <int B>
+__host__ __device__ constexpr uint32_t unshift_h2(int rho) {
+  return (((uint32_t)(Window<B>::k(rho) - Window<B>::kmin() + 15) << 10) * 0x00010001u);
+}
+
 // V side: add one code row's rank-space contribution into the shared-memory accumulators.
+// The tile holding strip P = r/2 is always processed: its lanes on strip P feed the constant
+// rows r (code 0, i.e. 1.0: zero words) and r + 1 (the per-register window factor).
 template <int G, int B>
 __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, const uint32_t (&bv)[8][2],
                                                  uint32_t one, float* osm) {
   constexpr int NO = OAcc<G>::N;
   const int lane = threadIdx.x & 31;
   const int P = rv >> 1;
-  const int nfull = P >> 3, nmu = (P + 7) >> 3;
+  const int nfull = P >> 3;
   // lane's pieces: strips 8 mu + (lane >> 3) and + 4, piece lane & 7
   const uint8_t* pa = stage + (lane >> 3) * 32 * B + (lane & 7) * 4 * B;
   float* o = osm + lane * NO;
   auto tile = [&](bool check, int mu) {
-    // rows for channels past r are never written out, so their operand values only need to
-    // be finite
     uint32_t wa[B], wb[B];
+    bool la = false, lb = false;  // this lane feeds the normaliser row (strip P, odd channel)
     if (check) {
       const int sA = 8 * mu + (lane >> 3);
       load_piece_or_zero<B>(pa, sA < P, wa);
       load_piece_or_zero<B>(pa + 4 * 32 * B, sA + 4 < P, wb);
+      la = B <= 2 && sA == P && (lane & 4);
+      lb = B <= 2 && sA + 4 == P && (lane & 4);
     } else {
       load_piece<B>(pa, wa);
       load_piece<B>(pa + 4 * 32 * B, wb);
@@ -314,8 +329,16 @@ __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, c
     float d[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
-      const uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wb, 2 * t, one);
-      const uint32_t a2 = unpack_reg<B>(wa, 2 * t + 1, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
+      uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wb, 2 * t, one);
+      uint32_t a2 = unpack_reg<B>(wa, 2 * t + 1, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
+      if constexpr (B <= 2) {
+        if (check) {
+          a0 = la ? unshift_h2<B>(2 * t) : a0;
+          a2 = la ? unshift_h2<B>(2 * t + 1) : a2;
+          a1 = lb ? unshift_h2<B>(2 * t) : a1;
+          a3 = lb ? unshift_h2<B>(2 * t + 1) : a3;
+        }
+      }
       mma_f16(d[t & 1], a0, a1, a2, a3, bv[t][0], bv[t][1]);
     }
     if constexpr (NO == 2) {
@@ -336,7 +359,7 @@ __device__ __forceinline__ void v_row_accumulate(const uint8_t* stage, int rv, c
   };
 #pragma unroll 1
   for (int mu = 0; mu < nfull; ++mu) tile(false, mu);
-  if (nmu > nfull) tile(true, nfull);
+  tile(true, nfull);
 }
 
 template <int G>
@@ -355,6 +378,7 @@ __device__ __forceinline__ void k_row_dispatch(int b, const uint8_t* stage, int 
   }
 }
 
+// b = 0 stands for a head with r_V = 0: only the constant rows (one window class)
 template <int G>
 __device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int rv, const uint32_t (&bv)[8][2],
                                                uint32_t one, float* osm) {
@@ -366,71 +390,45 @@ __device__ __forceinline__ void v_row_dispatch(int b, const uint8_t* stage, int 
     case 5: v_row_accumulate<G, 5>(stage, rv, bv, one, osm); break;
     case 6: v_row_accumulate<G, 6>(stage, rv, bv, one, osm); break;
     case 7: v_row_accumulate<G, 7>(stage, rv, bv, one, osm); break;
-    default: v_row_accumulate<G, 8>(stage, rv, bv, one, osm); break;
+    case 8: v_row_accumulate<G, 8>(stage, rv, bv, one, osm); break;
+    default: v_row_accumulate<G, 3>(stage, 0, bv, one, osm); break;
   }
 }
 
 template <int G>
-__device__ __forceinline__ size_t decode_osm_bytes() {
-  return (size_t)8 * 32 * OAcc<G>::N * sizeof(float);
+__host__ __device__ constexpr size_t decode_osm_bytes() {
+  return (size_t)kMaxVTiles * 32 * OAcc<G>::N * sizeof(float);
 }
 
-// Online softmax of one row's scores (base 2) and the V-side MMA operands.  VC is the V bit
-// width's window class: 0 = one window for every register (b >= 3), 1 or 2 = the b = 1 / b = 2
-// windows.  V codes read 1 + code * 2^(k-10) with a per-register window k, so each token's
-// probability is fed to the MMA pre-scaled by 2^(kmin - k) (folded into the exponent): the
-// products then carry the single scale 2^(kmin-10), and the unit offsets add up to the plain
-// sum of the fed values, accumulated in c.  Every fed value is rounded to fp16 once and the
-// same rounded value enters l, c and the MMA, so the weights stay exactly normalised.
+// VC is the V bit width's window class: 0 = one window for every register (b >= 3, or no V
+// codes), 1 or 2 = the b = 1 / b = 2 windows.  V codes read 1 + code * 2^(k-10) with a
+// per-register window k, so each token's probability is fed to the MMA pre-scaled by
+// 2^(kmin - k) (folded into the exponent): the products then carry the single scale
+// 2^(kmin-10), and the unit offsets add up to the plain sum of the fed values.
 template <int VC>
 struct VWin {
   static constexpr int B = VC == 0 ? 3 : VC;
   __device__ static constexpr float shift(int rho) {  // kmin - k (<= 0)
     return VC == 0 ? 0.f : (float)(Window<B>::kmin() - Window<B>::k(rho));
   }
-  __device__ static constexpr float unshift(int rho) {  // 2^(k - kmin)
-    return VC == 0 ? 1.f : (float)(1 << (Window<B>::k(rho) - Window<B>::kmin()));
-  }
 };
 
+// Probabilities of one row against the reference max, as the V side's MMA B operands: the
+// 16 x 8 probability tile of token tile t in C-fragment layout (row t0 or t1, columns 2j,
+// 2j+1), transposed by movmatrix.  Each fed value is rounded to fp16 once; the same value
+// enters O, c and l through the MMA, so the weights stay exactly normalised.
 template <int G, int VC>
-__device__ __forceinline__ void row_softmax(float (&s)[8][G / 4][2], WarpState<G>& st, float (&alpha)[G / 4],
-                                            bool& rescale, uint32_t (&bv)[8][2]) {
+__device__ __forceinline__ void row_probs(const float (&s)[8][G / 4][2], const float (&mref)[G / 4],
+                                          uint32_t (&bv)[8][2]) {
   constexpr int NG = G / 4;
   float pf[8][NG][2];
 #pragma unroll
-  for (int u = 0; u < NG; ++u) {
-    float mx = -INFINITY;
-#pragma unroll
-    for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][u][0], s[t][u][1]));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-    const float mnew = fmaxf(st.m[u], mx);
-    alpha[u] = ex2_approx(st.m[u] - mnew);
-    rescale |= (mnew != st.m[u]);
-    st.m[u] = mnew;
-    float ls = 0.f, cs = 0.f;
+  for (int u = 0; u < NG; ++u)
 #pragma unroll
     for (int t = 0; t < 8; ++t) {
-      const float e0 = s[t][u][0] - mnew + VWin<VC>::shift(2 * t);
-      const float e1 = s[t][u][1] - mnew + VWin<VC>::shift(2 * t + 1);
-      const float2 q = __half22float2(__floats2half2_rn(ex2_approx(e0), ex2_approx(e1)));
-      pf[t][u][0] = q.x;
-      pf[t][u][1] = q.y;
-      if constexpr (VC == 0) {
-        ls += q.x + q.y;
-      } else {
-        ls += q.x * VWin<VC>::unshift(2 * t) + q.y * VWin<VC>::unshift(2 * t + 1);
-        cs += q.x + q.y;
-      }
+      pf[t][u][0] = ex2_approx(s[t][u][0] + (VWin<VC>::shift(2 * t) - mref[u]));
+      pf[t][u][1] = ex2_approx(s[t][u][1] + (VWin<VC>::shift(2 * t + 1) - mref[u]));
     }
-    st.l[u] = st.l[u] * alpha[u] + ls;
-    st.c[u] = st.c[u] * alpha[u] + cs;
-  }
-  // B fragments of the V side: the 16 x 8 probability tile of token tile t in C-fragment
-  // layout (row t0 or t1, columns 2j, 2j+1), transposed by movmatrix.  The fp16 values are
-  // exact (they were rounded above).
 #pragma unroll
   for (int t = 0; t < 8; ++t) {
     const float c0 = pf[t][0][0], c1 = NG == 2 ? pf[t][NG - 1][0] : 0.f;
@@ -445,12 +443,13 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
   constexpr int NG = G / 4, NO = OAcc<G>::N;
   extern __shared__ __align__(128) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool leader = lane == 0;
   const int ring_bytes = a.ring_bytes;
   const size_t warp_bytes = (size_t)ring_bytes + decode_osm_bytes<G>();
   uint8_t* ring = smem + (size_t)warp * warp_bytes;
   float* osm = reinterpret_cast<float*>(ring + ring_bytes);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)kDecodeWarps * warp_bytes) + warp * kMaxStages;
-  if (lane == 0) {
+  if (leader) {
     for (int i = 0; i < kMaxStages; ++i) mbar_init(smem_addr(&bars[i]), 1);
     fence_mbar_init();
   }
@@ -465,15 +464,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
   const int gstride = wh->g_stride, pstride = wh->part_stride;
   uint32_t phase_bits = 0;  // parity of the next wait per barrier
   bool failed = false;
-  int outstanding = 0;      // loads issued but not yet waited for
-  int wait_stage = 0, nstage = 2;
+  int outstanding = 0;      // stages issued but not yet waited for
+  int wait_stage = 0, nstage = 1;
 
   // work items are taken in plan order from a shared counter, so that warps that finish early
   // take more (the items' costs differ with the heads' bit widths)
   unsigned int* next_item = const_cast<unsigned int*>(&wh->next_item);
   auto take = [&]() -> int {
     int v = 0;
-    if (lane == 0) v = (int)atomicAdd(next_item, 1u);
+    if (leader) v = (int)atomicAdd(next_item, 1u);
     return __shfl_sync(0xffffffffu, v, 0);
   };
   for (int item = take(); item < n_items && !failed; item = take()) {
@@ -486,36 +485,33 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     const int row0 = it.row_begin, row1 = min(it.row_end, rows_valid);
     float* part = parts + (size_t)item * pstride;
     const uint32_t rbk = kr > 0 ? 16u * kr * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
-    // this item's stages: as many buffers of its largest row as the ring holds (every load of
-    // the previous item has been consumed, so the ring is free)
-    const int stage_bytes = (int)((max(max(rbk, rbv), 16u) + 127u) & ~127u);
+    // one stage = this item's K row + V row (every load of the previous item has been
+    // consumed, so the whole ring is free)
+    const uint32_t kst = (rbk + 127u) & ~127u;
+    const int stage_bytes = (int)max(kst + ((rbv + 127u) & ~127u), 128u);
     nstage = min(kMaxStages, ring_bytes / stage_bytes);
     wait_stage = 0;
-    if (nstage < 2) {
-      // a row that does not fit the staging buffer is never copied; report and leave an
+    if (nstage < 1) {
+      // a row pair that does not fit the staging ring is never copied; report and leave an
       // empty chunk (m = -inf, l = 0)
-      if (lane == 0) atomicOr(&g_status, 2u);
+      if (leader) atomicOr(&g_status, 2u);
       if (lane < G) {
         part[lane * gstride + 0] = -INFINITY;
         part[lane * gstride + 1] = 0.f;
       }
       continue;
     }
-    WarpState<G> st;
+    float mref[NG];
 #pragma unroll
-    for (int u = 0; u < NG; ++u) {
-      st.m[u] = -INFINITY;
-      st.l[u] = 0.f;
-      st.c[u] = 0.f;
-    }
-    const int nmu = ((vr >> 1) + 7) >> 3;
-    for (int k = 0; k < nmu * NO; ++k) osm[k * 32 + lane] = 0.f;
-    // V window class (see row_softmax) and the factor 2^(10 - kmin) that turns the fed
-    // products back into codes
+    for (int u = 0; u < NG; ++u) mref[u] = -INFINITY;
+    const int ntile = (vr >> 4) + 1;  // V accumulator tiles incl. the constant rows
+    for (int k = 0; k < ntile * NO; ++k) osm[k * 32 + lane] = 0.f;
+    // V window class (see VWin) and the factor 2^(10 - kmin) that turns the fed products back
+    // into codes
     const int vc = (vr > 0 && vb <= 2) ? vb : 0;
+    const int vbd = vr > 0 ? vb : 0;
     const float vout = vr == 0 ? 0.f : (float)(1 << (vb == 1 ? 5 : vb == 2 ? 6 : vb));
-    const bool two = rbk && rbv;
-    const int n_loads = row1 > row0 ? (row1 - row0) * (two ? 2 : (rbk || rbv ? 1 : 0)) : 0;
+    const int n_loads = (row1 > row0 && (rbk || rbv)) ? row1 - row0 : 0;
     const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
     const float* qhdr = reinterpret_cast<const float*>(qt);
     const uint2* bfrag = reinterpret_cast<const uint2*>(qt + kQtHeaderBytes);
@@ -525,29 +521,27 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     const float qscale = qhdr[8];
     const uint32_t one = a.one;
 
-    // issue state (lane 0 only): next row / side / stage to load
+    // issue state: next row and stage to load (every lane tracks it; lane 0 issues)
     int iss_row = row0, iss_stage = 0;
-    bool iss_v = !rbk;
     const uint8_t* kbase = a.cache + koff;
     const uint8_t* vbase = a.cache + voff;
     auto issue_next = [&]() {
-      const uint32_t bytes = iss_v ? rbv : rbk;
-      const uint8_t* src = (iss_v ? vbase : kbase) +
-                           row_offset(0, bytes, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq);
       const uint32_t bar = smem_addr(&bars[iss_stage]);
-      mbar_arrive_expect_tx(bar, bytes);
-      bulk_g2s(smem_addr(ring + (size_t)iss_stage * stage_bytes), src, bytes, bar);
-      if (two && !iss_v) {
-        iss_v = true;
-      } else {
-        iss_v = !rbk;
-        ++iss_row;
-      }
+      const uint32_t dst = smem_addr(ring + (size_t)iss_stage * stage_bytes);
+      mbar_arrive_expect_tx_if(leader, bar, rbk + rbv);
+      if (rbk)
+        bulk_g2s_if(leader, dst,
+                    kbase + row_offset(0, rbk, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbk,
+                    bar);
+      if (rbv)
+        bulk_g2s_if(leader, dst + kst,
+                    vbase + row_offset(0, rbv, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbv,
+                    bar);
+      ++iss_row;
       if (++iss_stage == nstage) iss_stage = 0;
     };
     int issued = min(n_loads, nstage);
-    if (lane == 0)
-      for (int k = 0; k < issued; ++k) issue_next();
+    for (int k = 0; k < issued; ++k) issue_next();
     outstanding = issued;
 
     // wait for the next stage; returns its buffer or nullptr on timeout
@@ -558,32 +552,31 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       phase_bits ^= 1u << wait_stage;
       return ring + (size_t)wait_stage * stage_bytes;
     };
-    // release the stage just consumed and refill it with the next load of this item
+    // release the stage just consumed and refill it with the next row pair of this item
     auto release = [&]() {
       __syncwarp();
       --outstanding;
       if (++wait_stage == nstage) wait_stage = 0;
       if (issued < n_loads) {
-        if (lane == 0) {
-          fence_proxy_async_smem();
-          issue_next();
-        }
+        fence_proxy_async_smem_if(leader);
+        issue_next();
         ++issued;
         ++outstanding;
       }
     };
 
     for (int row = row0; row < row1; ++row) {
-      float s[8][NG][2];
-      // ---- K row ----
-      if (rbk) {
-        const uint8_t* buf = acquire();
+      const uint8_t* buf = nullptr;
+      if (n_loads) {
+        buf = acquire();
         if (!buf) {
           failed = true;
           break;
         }
+      }
+      float s[8][NG][2];
+      if (rbk) {
         k_row_dispatch<G>(kb, buf, kr, bfrag, qsum, qscale, one, s);
-        release();
       } else {
 #pragma unroll
         for (int t = 0; t < 8; ++t)
@@ -600,53 +593,60 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
             if (tbase + 16 * t + 8 >= T) s[t][u][1] = -INFINITY;
           }
       }
-      uint32_t bv[8][2];
-      bool rescale = false;
+      // row max per head; the reference max moves (and the accumulators are rescaled) only
+      // when it is exceeded by more than kTau
+      bool move = false;
       float alpha[NG];
-      if (vc == 1)
-        row_softmax<G, 1>(s, st, alpha, rescale, bv);
-      else if (vc == 2)
-        row_softmax<G, 2>(s, st, alpha, rescale, bv);
-      else
-        row_softmax<G, 0>(s, st, alpha, rescale, bv);
-      // ---- V row ----
-      if (rbv) {
-        if (__any_sync(0xffffffffu, rescale)) {
-          for (int mu = 0; mu < nmu; ++mu) {
-            float* o = osm + (mu * 32 + lane) * NO;
 #pragma unroll
-            for (int k = 0; k < NO; ++k) o[k] *= alpha[NG == 2 ? (k & 1) : 0];
-          }
-        }
-        const uint8_t* buf = acquire();
-        if (!buf) {
-          failed = true;
-          break;
-        }
-        v_row_dispatch<G>(vb, buf, vr, bv, one, osm);
-        release();
+      for (int u = 0; u < NG; ++u) {
+        float mx = -INFINITY;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][u][0], s[t][u][1]));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        const bool mv = mx > mref[u] + kTau;
+        alpha[u] = mv ? ex2_approx(mref[u] - mx) : 1.f;
+        mref[u] = mv ? mx : mref[u];
+        move |= mv;
       }
+      if (__any_sync(0xffffffffu, move)) {
+        for (int mu = 0; mu < ntile; ++mu) {
+          float* o = osm + (mu * 32 + lane) * NO;
+#pragma unroll
+          for (int k = 0; k < NO; ++k) o[k] *= alpha[NG == 2 ? (k & 1) : 0];
+        }
+      }
+      uint32_t bv[8][2];
+      if (vc == 1)
+        row_probs<G, 1>(s, mref, bv);
+      else if (vc == 2)
+        row_probs<G, 2>(s, mref, bv);
+      else
+        row_probs<G, 0>(s, mref, bv);
+      v_row_dispatch<G>(vbd, buf + kst, vr, bv, one, osm);
+      if (n_loads) release();
     }
     if (failed) break;
-    // ---- write the partial of this item ----
+    // ---- write the partial of this item: m, l and (O - c) 2^(10 - kmin) per query head ----
     __syncwarp();
+    const int cr = vr & 15, ct = vr >> 4;  // constant rows r, r + 1: tile ct, rows cr, cr + 1
 #pragma unroll
     for (int u = 0; u < NG; ++u) {
-      float l = st.l[u], c = st.c[u];
-      l += __shfl_xor_sync(0xffffffffu, l, 4);
-      l += __shfl_xor_sync(0xffffffffu, l, 8);
-      l += __shfl_xor_sync(0xffffffffu, l, 16);
-      c += __shfl_xor_sync(0xffffffffu, c, 4);
-      c += __shfl_xor_sync(0xffffffffu, c, 8);
-      c += __shfl_xor_sync(0xffffffffu, c, 16);
-      if (vc == 0) c = l;
       const int g = Heads<G>::head(lane & 3, u);
+      // entry of (row, head g) in a tile: lane 4 (row % 8) + column owner, slot by row half
+      auto at = [&](int row) -> float {
+        const int ln = 4 * (row & 7) + (G == 4 ? g : (g >> 1));
+        const int sl = G == 4 ? ((row >> 3) & 1) : 2 * ((row >> 3) & 1) + (g & 1);
+        return osm[(ct * 32 + ln) * NO + sl];
+      };
+      const float c = at(cr), l = at(cr + 1);
       float* pg = part + g * gstride;
       if ((lane >> 2) == 0) {
-        pg[0] = st.m[u];
+        pg[0] = mref[u];
         pg[1] = l;
       }
-      for (int mu = 0; mu < nmu; ++mu) {
+      for (int mu = 0; mu < ntile; ++mu) {
         const float* o = osm + (mu * 32 + lane) * NO;
         // G = 4: [ch0, ch1]; G = 8: [ch0 head 2j, ch0 head 2j+1, ch1 head 2j, ch1 head 2j+1]
         const float o0 = NO == 2 ? o[0] : o[u], o1 = NO == 2 ? o[1] : o[2 + u];
@@ -658,7 +658,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     __syncwarp();
   }
   if (failed) {
-    if (lane == 0) atomicOr(&g_status, 1u);
+    if (leader) atomicOr(&g_status, 1u);
     // drain the copies still in flight before the shared memory goes away
     for (int k = 0; k < outstanding; ++k) {
       if (!mbar_wait_bounded(smem_addr(&bars[wait_stage]), (phase_bits >> wait_stage) & 1u, kWaitLimitNs)) break;

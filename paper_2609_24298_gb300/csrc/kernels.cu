@@ -206,7 +206,7 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
 }
 
 namespace {
-size_t decode_osm_bytes_host(int G) { return (size_t)8 * 32 * (G == 4 ? 2 : 4) * sizeof(float); }
+size_t decode_osm_bytes_host(int G) { return G == 4 ? decode_osm_bytes<4>() : decode_osm_bytes<8>(); }
 
 enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
