@@ -75,6 +75,15 @@ __device__ __forceinline__ void mbar_arrive_expect_tx_if(bool p, uint32_t bar, u
       "r"(bytes), "r"((int)p)
       : "memory");
 }
+// adds expected bytes to the current phase without arriving (the arrival comes with a later
+// arrive.expect_tx on the same barrier)
+__device__ __forceinline__ void mbar_expect_tx_if(bool p, uint32_t bar, uint32_t bytes) {
+  asm volatile(
+      "{\n .reg .pred q;\n setp.ne.b32 q, %2, 0;\n @q mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;\n}\n" ::"r"(
+          bar),
+      "r"(bytes), "r"((int)p)
+      : "memory");
+}
 __device__ __forceinline__ void bulk_g2s_if(bool p, uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
   asm volatile(
       "{\n .reg .pred q;\n setp.ne.b32 q, %4, 0;\n"

@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
           }
           e4[u] = v;
         }
-        frag[(kap * 2 + nt) * 32 + fl] = make_uint2(pack_f16(e4[0], e4[1]), pack_f16(e4[2], e4[3]));
+        frag[(kap * NTK + nt) * 32 + fl] = make_uint2(pack_f16(e4[0], e4[1]), pack_f16(e4[2], e4[3]));
       }
     }
   }
@@ -263,7 +263,7 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
       for (int nt = 0; nt < NTK; ++nt) mma_f16(acc[t][nt], a0, a1, a2, a3, bf[nt].x, bf[nt].y);
     }
     pa += 8 * 32 * B;
-    bq += 2 * 32;
+    bq += NTK * 32;
   };
 #pragma unroll 1
   for (int kap = 0; kap < nfull; ++kap) tile(false, kap);
@@ -399,6 +399,11 @@ template <int G>
 __host__ __device__ constexpr size_t decode_osm_bytes() {
   return (size_t)kMaxVTiles * 32 * OAcc<G>::N * sizeof(float);
 }
+// the group's q~ MMA B fragments, copied into the warp's shared memory once per work item
+template <int G>
+__host__ __device__ constexpr uint32_t decode_qfrag_bytes() {
+  return 8u * Heads<G>::NTK * 32u * 8u;
+}
 
 // VC is the V bit width's window class: 0 = one window for every register (b >= 3, or no V
 // codes), 1 or 2 = the b = 1 / b = 2 windows.  V codes read 1 + code * 2^(k-10) with a
@@ -438,19 +443,251 @@ __device__ __forceinline__ void row_probs(const float (&s)[8][G / 4][2], const f
   }
 }
 
+// Per-warp state of the scan that outlives a work item.
+struct ScanWarp {
+  uint8_t* ring;
+  float* osm;
+  uint2* qfrag;
+  uint64_t* bars;
+  int ring_bytes, lane;
+  bool leader, failed;
+  uint32_t phase_bits;  // parity of the next wait per barrier
+  int wait_stage, nstage, outstanding;
+};
+
+// One work item.  BK / BV > 0 fix the K / V bit widths at compile time (the common widths
+// get their own copy of the row loop); 0 dispatches on the runtime widths row by row.
+template <int G, int BK, int BV>
+__device__ __forceinline__ void scan_item(const DecodeArgs& a, ScanWarp& w, int item) {
+  constexpr int NG = G / 4, NO = OAcc<G>::N;
+  const int lane = w.lane;
+  const bool leader = w.leader;
+  const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
+  const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
+  const WsItem* items = reinterpret_cast<const WsItem*>(a.ws + wh->items_off);
+  const HeadEntry* heads = head_table(a.block);
+  float* parts = reinterpret_cast<float*>(a.ws + wh->part_off);
+  const int gstride = wh->g_stride, pstride = wh->part_stride;
+  const WsItem it = items[item];
+  const WsGroup gr = groups[it.group];
+  const int kr = heads[gr.k_head].r, vr = heads[gr.v_head].r;
+  const int kb = BK > 0 ? BK : heads[gr.k_head].b, vb = BV > 0 ? BV : heads[gr.v_head].b;
+  const uint64_t koff = heads[gr.k_head].cache_off, voff = heads[gr.v_head].cache_off;
+  const int T = a.seq_lens[gr.seq];
+  const int rows_valid = (T + kRowTokens - 1) / kRowTokens;
+  const int row0 = it.row_begin, row1 = min(it.row_end, rows_valid);
+  float* part = parts + (size_t)item * pstride;
+  const uint32_t rbk = kr > 0 ? 16u * kr * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
+  // one stage = this item's K row + V row (every load of the previous item has been
+  // consumed, so the whole ring is free)
+  const uint32_t kst = (rbk + 127u) & ~127u;
+  const int stage_bytes = (int)max(kst + ((rbv + 127u) & ~127u), 128u);
+  w.nstage = min(kMaxStages, w.ring_bytes / stage_bytes);
+  w.wait_stage = 0;
+  if (w.nstage < 1) {
+    // a row pair that does not fit the staging ring is never copied; report and leave an
+    // empty chunk (m = -inf, l = 0)
+    if (leader) atomicOr(&g_status, 2u);
+    if (lane < G) {
+      part[lane * gstride + 0] = -INFINITY;
+      part[lane * gstride + 1] = 0.f;
+    }
+    return;
+  }
+  float* osm = w.osm;
+  float mref[NG];
+#pragma unroll
+  for (int u = 0; u < NG; ++u) mref[u] = -INFINITY;
+  const int ntile = (vr >> 4) + 1;  // V accumulator tiles incl. the constant rows
+  for (int k = 0; k < ntile * NO; ++k) osm[k * 32 + lane] = 0.f;
+  // V window class (see VWin) and the factor 2^(10 - kmin) that turns the fed products back
+  // into codes
+  const int vc = (vr > 0 && vb <= 2) ? vb : 0;
+  const int vbd = vr > 0 ? vb : 0;
+  const float vout = vr == 0 ? 0.f : (float)(1 << (vb == 1 ? 5 : vb == 2 ? 6 : vb));
+  const int n_loads = (row1 > row0 && (rbk || rbv)) ? row1 - row0 : 0;
+  const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
+  const float* qhdr = reinterpret_cast<const float*>(qt);
+  const uint2* bfrag = w.qfrag;  // filled together with the item's first stage
+  float qsum[NG];
+#pragma unroll
+  for (int u = 0; u < NG; ++u) qsum[u] = qhdr[Heads<G>::head(lane & 3, u)];
+  const float qscale = qhdr[8];
+  const uint32_t one = a.one;
+
+  // issue state: next row and stage to load (every lane tracks it; lane 0 issues)
+  int iss_row = row0, iss_stage = 0;
+  const uint8_t* kbase = a.cache + koff;
+  const uint8_t* vbase = a.cache + voff;
+  auto issue_next = [&]() {
+    const uint32_t bar = smem_addr(&w.bars[iss_stage]);
+    const uint32_t dst = smem_addr(w.ring + (size_t)iss_stage * stage_bytes);
+    mbar_arrive_expect_tx_if(leader, bar, rbk + rbv);
+    if (rbk)
+      bulk_g2s_if(leader, dst,
+                  kbase + row_offset(0, rbk, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbk,
+                  bar);
+    if (rbv)
+      bulk_g2s_if(leader, dst + kst,
+                  vbase + row_offset(0, rbv, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbv,
+                  bar);
+    ++iss_row;
+    if (++iss_stage == w.nstage) iss_stage = 0;
+  };
+  int issued = min(n_loads, w.nstage);
+  if (issued > 0 && rbk) {
+    // the q~ fragments travel with the first stage: the previous item's reads of them are
+    // ordered before the copy by the warp barrier and the proxy fence
+    __syncwarp();
+    fence_proxy_async_smem_if(leader);
+    const uint32_t bar = smem_addr(&w.bars[0]);
+    mbar_expect_tx_if(leader, bar, decode_qfrag_bytes<G>());  // stage 0's issue below arrives
+    bulk_g2s_if(leader, smem_addr(w.qfrag), qt + kQtHeaderBytes, decode_qfrag_bytes<G>(), bar);
+  }
+  for (int k = 0; k < issued; ++k) issue_next();
+  w.outstanding = issued;
+
+  // wait for the next stage; returns its buffer or nullptr on timeout
+  auto acquire = [&]() -> const uint8_t* {
+    const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&w.bars[w.wait_stage]),
+                                                              (w.phase_bits >> w.wait_stage) & 1u, kWaitLimitNs));
+    if (!ok) return nullptr;
+    w.phase_bits ^= 1u << w.wait_stage;
+    return w.ring + (size_t)w.wait_stage * stage_bytes;
+  };
+  // release the stage just consumed and refill it with the next row pair of this item
+  auto release = [&]() {
+    __syncwarp();
+    --w.outstanding;
+    if (++w.wait_stage == w.nstage) w.wait_stage = 0;
+    if (issued < n_loads) {
+      fence_proxy_async_smem_if(leader);
+      issue_next();
+      ++issued;
+      ++w.outstanding;
+    }
+  };
+
+  for (int row = row0; row < row1; ++row) {
+    const uint8_t* buf = nullptr;
+    if (n_loads) {
+      buf = acquire();
+      if (!buf) {
+        w.failed = true;
+        return;
+      }
+    }
+    float s[8][NG][2];
+    if (rbk) {
+      if constexpr (BK > 0)
+        k_row_scores<G, BK>(buf, kr, bfrag, qsum, qscale, one, s);
+      else
+        k_row_dispatch<G>(kb, buf, kr, bfrag, qsum, qscale, one, s);
+    } else {
+#pragma unroll
+      for (int t = 0; t < 8; ++t)
+#pragma unroll
+        for (int u = 0; u < NG; ++u) s[t][u][0] = s[t][u][1] = 0.f;
+    }
+    if ((row + 1) * kRowTokens > T) {  // only the last row of a sequence has masked tokens
+      const int tbase = row * kRowTokens + (lane >> 2);
+#pragma unroll
+      for (int u = 0; u < NG; ++u)
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+          if (tbase + 16 * t >= T) s[t][u][0] = -INFINITY;
+          if (tbase + 16 * t + 8 >= T) s[t][u][1] = -INFINITY;
+        }
+    }
+    // row max per head; the reference max moves (and the accumulators are rescaled) only
+    // when it is exceeded by more than kTau
+    bool move = false;
+    float alpha[NG];
+#pragma unroll
+    for (int u = 0; u < NG; ++u) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][u][0], s[t][u][1]));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+      const bool mv = mx > mref[u] + kTau;
+      alpha[u] = mv ? ex2_approx(mref[u] - mx) : 1.f;
+      mref[u] = mv ? mx : mref[u];
+      move |= mv;
+    }
+    if (__any_sync(0xffffffffu, move)) {
+      for (int mu = 0; mu < ntile; ++mu) {
+        float* o = osm + (mu * 32 + lane) * NO;
+#pragma unroll
+        for (int k = 0; k < NO; ++k) o[k] *= alpha[NG == 2 ? (k & 1) : 0];
+      }
+    }
+    uint32_t bv[8][2];
+    if constexpr (BV > 0) {
+      row_probs<G, (BV <= 2 ? BV : 0)>(s, mref, bv);
+      v_row_accumulate<G, BV>(buf + kst, vr, bv, one, osm);
+    } else {
+      if (vc == 1)
+        row_probs<G, 1>(s, mref, bv);
+      else if (vc == 2)
+        row_probs<G, 2>(s, mref, bv);
+      else
+        row_probs<G, 0>(s, mref, bv);
+      v_row_dispatch<G>(vbd, buf + kst, vr, bv, one, osm);
+    }
+    if (n_loads) release();
+  }
+  // ---- write the partial of this item: m, l and (O - c) 2^(10 - kmin) per query head ----
+  __syncwarp();
+  const int cr = vr & 15, ct = vr >> 4;  // constant rows r, r + 1: tile ct, rows cr, cr + 1
+#pragma unroll
+  for (int u = 0; u < NG; ++u) {
+    const int g = Heads<G>::head(lane & 3, u);
+    // entry of (row, head g) in a tile: lane 4 (row % 8) + column owner, slot by row half
+    auto at = [&](int row) -> float {
+      const int ln = 4 * (row & 7) + (G == 4 ? g : (g >> 1));
+      const int sl = G == 4 ? ((row >> 3) & 1) : 2 * ((row >> 3) & 1) + (g & 1);
+      return osm[(ct * 32 + ln) * NO + sl];
+    };
+    const float c = at(cr), l = at(cr + 1);
+    float* pg = part + g * gstride;
+    if ((lane >> 2) == 0) {
+      pg[0] = mref[u];
+      pg[1] = l;
+    }
+    for (int mu = 0; mu < ntile; ++mu) {
+      const float* o = osm + (mu * 32 + lane) * NO;
+      // G = 4: [ch0, ch1]; G = 8: [ch0 head 2j, ch0 head 2j+1, ch1 head 2j, ch1 head 2j+1]
+      const float o0 = NO == 2 ? o[0] : o[u], o1 = NO == 2 ? o[1] : o[2 + u];
+      const int ch0 = 16 * mu + (lane >> 2), ch1 = ch0 + 8;
+      if (ch0 < vr) pg[4 + ch0] = (o0 - c) * vout;
+      if (ch1 < vr) pg[4 + ch1] = (o1 - c) * vout;
+    }
+  }
+  __syncwarp();
+}
+
 template <int G>
 __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs a) {
-  constexpr int NG = G / 4, NO = OAcc<G>::N;
   extern __shared__ __align__(128) uint8_t smem[];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool leader = lane == 0;
-  const int ring_bytes = a.ring_bytes;
-  const size_t warp_bytes = (size_t)ring_bytes + decode_osm_bytes<G>();
-  uint8_t* ring = smem + (size_t)warp * warp_bytes;
-  float* osm = reinterpret_cast<float*>(ring + ring_bytes);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)kDecodeWarps * warp_bytes) + warp * kMaxStages;
-  if (leader) {
-    for (int i = 0; i < kMaxStages; ++i) mbar_init(smem_addr(&bars[i]), 1);
+  const int warp = threadIdx.x >> 5;
+  ScanWarp w;
+  w.lane = threadIdx.x & 31;
+  w.leader = w.lane == 0;
+  w.ring_bytes = a.ring_bytes;
+  const size_t warp_bytes = (size_t)w.ring_bytes + decode_osm_bytes<G>() + decode_qfrag_bytes<G>();
+  w.ring = smem + (size_t)warp * warp_bytes;
+  w.osm = reinterpret_cast<float*>(w.ring + w.ring_bytes);
+  w.qfrag = reinterpret_cast<uint2*>(w.ring + w.ring_bytes + decode_osm_bytes<G>());
+  w.bars = reinterpret_cast<uint64_t*>(smem + (size_t)kDecodeWarps * warp_bytes) + warp * kMaxStages;
+  w.failed = false;
+  w.phase_bits = 0;
+  w.wait_stage = 0;
+  w.nstage = 1;
+  w.outstanding = 0;
+  if (w.leader) {
+    for (int i = 0; i < kMaxStages; ++i) mbar_init(smem_addr(&w.bars[i]), 1);
     fence_mbar_init();
   }
   __syncwarp();
@@ -459,211 +696,45 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
   const WsItem* items = reinterpret_cast<const WsItem*>(a.ws + wh->items_off);
   const HeadEntry* heads = head_table(a.block);
-  float* parts = reinterpret_cast<float*>(a.ws + wh->part_off);
   const int n_items = wh->n_items;
-  const int gstride = wh->g_stride, pstride = wh->part_stride;
-  uint32_t phase_bits = 0;  // parity of the next wait per barrier
-  bool failed = false;
-  int outstanding = 0;      // stages issued but not yet waited for
-  int wait_stage = 0, nstage = 1;
-
   // work items are taken in plan order from a shared counter, so that warps that finish early
   // take more (the items' costs differ with the heads' bit widths)
   unsigned int* next_item = const_cast<unsigned int*>(&wh->next_item);
   auto take = [&]() -> int {
     int v = 0;
-    if (leader) v = (int)atomicAdd(next_item, 1u);
+    if (w.leader) v = (int)atomicAdd(next_item, 1u);
     return __shfl_sync(0xffffffffu, v, 0);
   };
-  for (int item = take(); item < n_items && !failed; item = take()) {
-    const WsItem it = items[item];
-    const WsGroup gr = groups[it.group];
-    const int kr = heads[gr.k_head].r, kb = heads[gr.k_head].b, vr = heads[gr.v_head].r, vb = heads[gr.v_head].b;
-    const uint64_t koff = heads[gr.k_head].cache_off, voff = heads[gr.v_head].cache_off;
-    const int T = a.seq_lens[gr.seq];
-    const int rows_valid = (T + kRowTokens - 1) / kRowTokens;
-    const int row0 = it.row_begin, row1 = min(it.row_end, rows_valid);
-    float* part = parts + (size_t)item * pstride;
-    const uint32_t rbk = kr > 0 ? 16u * kr * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
-    // one stage = this item's K row + V row (every load of the previous item has been
-    // consumed, so the whole ring is free)
-    const uint32_t kst = (rbk + 127u) & ~127u;
-    const int stage_bytes = (int)max(kst + ((rbv + 127u) & ~127u), 128u);
-    nstage = min(kMaxStages, ring_bytes / stage_bytes);
-    wait_stage = 0;
-    if (nstage < 1) {
-      // a row pair that does not fit the staging ring is never copied; report and leave an
-      // empty chunk (m = -inf, l = 0)
-      if (leader) atomicOr(&g_status, 2u);
-      if (lane < G) {
-        part[lane * gstride + 0] = -INFINITY;
-        part[lane * gstride + 1] = 0.f;
+  for (int item = take(); item < n_items && !w.failed; item = take()) {
+    if constexpr (G == 4) {
+      // the bit widths of 1 to 3 that carry most of the cache at low rates get their own code
+      const WsGroup gr = groups[items[item].group];
+      const HeadEntry hk = heads[gr.k_head], hv = heads[gr.v_head];
+      const int key = (hk.r > 0 ? hk.b : 0) * 16 + (hv.r > 0 ? hv.b : 0);
+      switch (key) {
+        case 0x11: scan_item<G, 1, 1>(a, w, item); break;
+        case 0x12: scan_item<G, 1, 2>(a, w, item); break;
+        case 0x13: scan_item<G, 1, 3>(a, w, item); break;
+        case 0x21: scan_item<G, 2, 1>(a, w, item); break;
+        case 0x22: scan_item<G, 2, 2>(a, w, item); break;
+        case 0x23: scan_item<G, 2, 3>(a, w, item); break;
+        case 0x31: scan_item<G, 3, 1>(a, w, item); break;
+        case 0x32: scan_item<G, 3, 2>(a, w, item); break;
+        case 0x33: scan_item<G, 3, 3>(a, w, item); break;
+        default: scan_item<G, 0, 0>(a, w, item); break;
       }
-      continue;
+    } else {
+      scan_item<G, 0, 0>(a, w, item);
     }
-    float mref[NG];
-#pragma unroll
-    for (int u = 0; u < NG; ++u) mref[u] = -INFINITY;
-    const int ntile = (vr >> 4) + 1;  // V accumulator tiles incl. the constant rows
-    for (int k = 0; k < ntile * NO; ++k) osm[k * 32 + lane] = 0.f;
-    // V window class (see VWin) and the factor 2^(10 - kmin) that turns the fed products back
-    // into codes
-    const int vc = (vr > 0 && vb <= 2) ? vb : 0;
-    const int vbd = vr > 0 ? vb : 0;
-    const float vout = vr == 0 ? 0.f : (float)(1 << (vb == 1 ? 5 : vb == 2 ? 6 : vb));
-    const int n_loads = (row1 > row0 && (rbk || rbv)) ? row1 - row0 : 0;
-    const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
-    const float* qhdr = reinterpret_cast<const float*>(qt);
-    const uint2* bfrag = reinterpret_cast<const uint2*>(qt + kQtHeaderBytes);
-    float qsum[NG];
-#pragma unroll
-    for (int u = 0; u < NG; ++u) qsum[u] = qhdr[Heads<G>::head(lane & 3, u)];
-    const float qscale = qhdr[8];
-    const uint32_t one = a.one;
-
-    // issue state: next row and stage to load (every lane tracks it; lane 0 issues)
-    int iss_row = row0, iss_stage = 0;
-    const uint8_t* kbase = a.cache + koff;
-    const uint8_t* vbase = a.cache + voff;
-    auto issue_next = [&]() {
-      const uint32_t bar = smem_addr(&bars[iss_stage]);
-      const uint32_t dst = smem_addr(ring + (size_t)iss_stage * stage_bytes);
-      mbar_arrive_expect_tx_if(leader, bar, rbk + rbv);
-      if (rbk)
-        bulk_g2s_if(leader, dst,
-                    kbase + row_offset(0, rbk, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbk,
-                    bar);
-      if (rbv)
-        bulk_g2s_if(leader, dst + kst,
-                    vbase + row_offset(0, rbv, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbv,
-                    bar);
-      ++iss_row;
-      if (++iss_stage == nstage) iss_stage = 0;
-    };
-    int issued = min(n_loads, nstage);
-    for (int k = 0; k < issued; ++k) issue_next();
-    outstanding = issued;
-
-    // wait for the next stage; returns its buffer or nullptr on timeout
-    auto acquire = [&]() -> const uint8_t* {
-      const bool ok = __all_sync(
-          0xffffffffu, mbar_wait_bounded(smem_addr(&bars[wait_stage]), (phase_bits >> wait_stage) & 1u, kWaitLimitNs));
-      if (!ok) return nullptr;
-      phase_bits ^= 1u << wait_stage;
-      return ring + (size_t)wait_stage * stage_bytes;
-    };
-    // release the stage just consumed and refill it with the next row pair of this item
-    auto release = [&]() {
-      __syncwarp();
-      --outstanding;
-      if (++wait_stage == nstage) wait_stage = 0;
-      if (issued < n_loads) {
-        fence_proxy_async_smem_if(leader);
-        issue_next();
-        ++issued;
-        ++outstanding;
-      }
-    };
-
-    for (int row = row0; row < row1; ++row) {
-      const uint8_t* buf = nullptr;
-      if (n_loads) {
-        buf = acquire();
-        if (!buf) {
-          failed = true;
-          break;
-        }
-      }
-      float s[8][NG][2];
-      if (rbk) {
-        k_row_dispatch<G>(kb, buf, kr, bfrag, qsum, qscale, one, s);
-      } else {
-#pragma unroll
-        for (int t = 0; t < 8; ++t)
-#pragma unroll
-          for (int u = 0; u < NG; ++u) s[t][u][0] = s[t][u][1] = 0.f;
-      }
-      if ((row + 1) * kRowTokens > T) {  // only the last row of a sequence has masked tokens
-        const int tbase = row * kRowTokens + (lane >> 2);
-#pragma unroll
-        for (int u = 0; u < NG; ++u)
-#pragma unroll
-          for (int t = 0; t < 8; ++t) {
-            if (tbase + 16 * t >= T) s[t][u][0] = -INFINITY;
-            if (tbase + 16 * t + 8 >= T) s[t][u][1] = -INFINITY;
-          }
-      }
-      // row max per head; the reference max moves (and the accumulators are rescaled) only
-      // when it is exceeded by more than kTau
-      bool move = false;
-      float alpha[NG];
-#pragma unroll
-      for (int u = 0; u < NG; ++u) {
-        float mx = -INFINITY;
-#pragma unroll
-        for (int t = 0; t < 8; ++t) mx = fmaxf(mx, fmaxf(s[t][u][0], s[t][u][1]));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-        const bool mv = mx > mref[u] + kTau;
-        alpha[u] = mv ? ex2_approx(mref[u] - mx) : 1.f;
-        mref[u] = mv ? mx : mref[u];
-        move |= mv;
-      }
-      if (__any_sync(0xffffffffu, move)) {
-        for (int mu = 0; mu < ntile; ++mu) {
-          float* o = osm + (mu * 32 + lane) * NO;
-#pragma unroll
-          for (int k = 0; k < NO; ++k) o[k] *= alpha[NG == 2 ? (k & 1) : 0];
-        }
-      }
-      uint32_t bv[8][2];
-      if (vc == 1)
-        row_probs<G, 1>(s, mref, bv);
-      else if (vc == 2)
-        row_probs<G, 2>(s, mref, bv);
-      else
-        row_probs<G, 0>(s, mref, bv);
-      v_row_dispatch<G>(vbd, buf + kst, vr, bv, one, osm);
-      if (n_loads) release();
-    }
-    if (failed) break;
-    // ---- write the partial of this item: m, l and (O - c) 2^(10 - kmin) per query head ----
-    __syncwarp();
-    const int cr = vr & 15, ct = vr >> 4;  // constant rows r, r + 1: tile ct, rows cr, cr + 1
-#pragma unroll
-    for (int u = 0; u < NG; ++u) {
-      const int g = Heads<G>::head(lane & 3, u);
-      // entry of (row, head g) in a tile: lane 4 (row % 8) + column owner, slot by row half
-      auto at = [&](int row) -> float {
-        const int ln = 4 * (row & 7) + (G == 4 ? g : (g >> 1));
-        const int sl = G == 4 ? ((row >> 3) & 1) : 2 * ((row >> 3) & 1) + (g & 1);
-        return osm[(ct * 32 + ln) * NO + sl];
-      };
-      const float c = at(cr), l = at(cr + 1);
-      float* pg = part + g * gstride;
-      if ((lane >> 2) == 0) {
-        pg[0] = mref[u];
-        pg[1] = l;
-      }
-      for (int mu = 0; mu < ntile; ++mu) {
-        const float* o = osm + (mu * 32 + lane) * NO;
-        // G = 4: [ch0, ch1]; G = 8: [ch0 head 2j, ch0 head 2j+1, ch1 head 2j, ch1 head 2j+1]
-        const float o0 = NO == 2 ? o[0] : o[u], o1 = NO == 2 ? o[1] : o[2 + u];
-        const int ch0 = 16 * mu + (lane >> 2), ch1 = ch0 + 8;
-        if (ch0 < vr) pg[4 + ch0] = (o0 - c) * vout;
-        if (ch1 < vr) pg[4 + ch1] = (o1 - c) * vout;
-      }
-    }
-    __syncwarp();
   }
-  if (failed) {
-    if (leader) atomicOr(&g_status, 1u);
+  if (w.failed) {
+    if (w.leader) atomicOr(&g_status, 1u);
     // drain the copies still in flight before the shared memory goes away
-    for (int k = 0; k < outstanding; ++k) {
-      if (!mbar_wait_bounded(smem_addr(&bars[wait_stage]), (phase_bits >> wait_stage) & 1u, kWaitLimitNs)) break;
-      phase_bits ^= 1u << wait_stage;
-      if (++wait_stage == nstage) wait_stage = 0;
+    for (int k = 0; k < w.outstanding; ++k) {
+      if (!mbar_wait_bounded(smem_addr(&w.bars[w.wait_stage]), (w.phase_bits >> w.wait_stage) & 1u, kWaitLimitNs))
+        break;
+      w.phase_bits ^= 1u << w.wait_stage;
+      if (++w.wait_stage == w.nstage) w.wait_stage = 0;
     }
   }
 }

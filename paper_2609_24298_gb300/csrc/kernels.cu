@@ -206,7 +206,6 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
 }
 
 namespace {
-size_t decode_osm_bytes_host(int G) { return G == 4 ? decode_osm_bytes<4>() : decode_osm_bytes<8>(); }
 
 enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
@@ -226,7 +225,8 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_items, int st
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kScan) {
-    const size_t smem = (size_t)kDecodeWarps * ((size_t)a.ring_bytes + decode_osm_bytes_host(G) + kMaxStages * 8);
+    const size_t smem =
+        (size_t)kDecodeWarps * ((size_t)a.ring_bytes + decode_osm_bytes<G>() + decode_qfrag_bytes<G>() + kMaxStages * 8);
     static size_t attr_set = 0;
     if (smem > attr_set) {
       if (cudaFuncSetAttribute(decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
