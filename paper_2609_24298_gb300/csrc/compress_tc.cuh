@@ -4,16 +4,21 @@
 //
 // One CTA per (layer, kv head) and chunk of 128-token tiles, 6 warps:
 //   warp 0    TMA producer: each tile X [128 tokens x 128 dims] bf16 arrives as two 64-dim
-//             boxes with 128-byte swizzle into a 2-stage shared-memory ring.
-//   warp 1    allocates TMEM; one thread issues tcgen05.mma (M = 128 tokens, N = r padded to
-//             16, K = 16 per instruction, bf16 inputs, fp32 accumulation in TMEM) against the
-//             head's basis, which the CTA splits once into 2 (b <= 5) or 3 (b >= 6) bf16
-//             terms W = W0 + W1 (+ W2) held in shared memory in the same swizzled K-major
-//             layout: Y = X W0 + X W1 (+ X W2) reproduces the fp32 projection.  Two TMEM
+//             boxes with 128-byte swizzle into a 3-stage shared-memory ring.
+//   warp 1    allocates TMEM; one thread issues tcgen05.mma computing the transposed
+//             projection Y^T = W X^T (M = 128 channels, rows past r zero; N = 128 tokens;
+//             K = 16 per instruction; bf16 inputs, fp32 accumulation in TMEM).  The head's
+//             fp32 basis is split once per CTA into 2 (b <= 5) or 3 (b >= 6) bf16 terms
+//             W = W0 + W1 (+ W2) held in shared memory in the same swizzled K-major layout as
+//             X, so W0 X^T + W1 X^T (+ W2 X^T) reproduces the fp32 projection.  Two TMEM
 //             accumulators alternate between tiles.
-//   warps 2-5 epilogue: each reads its 32 TMEM lanes (tokens), subtracts W^T mu, quantises,
-//             writes the codes into a shared tile, and the four warps pack whole code rows
-//             with 32-bit stores.
+//   warps 2-5 epilogue: a thread owns one channel (its TMEM lane) and reads the 128 token
+//             values of its row of Y^T.  Token t's code goes to bits [(t/8) b, (t/8) b + b)
+//             of the channel's sub-stream t % 8, which is exactly where format v1 keeps it
+//             (K rows: piece t % 8, code rho = t / 8, half = channel parity; V rows: piece
+//             4 (channel parity) + (t/2) % 4, rho = t / 8, half = t % 2).  A lane then owns
+//             bytes [16 b i, 16 b (i + 1)) of the code row of its channel i: V rows from its
+//             own sub-streams, K rows after exchanging half of them with the partner channel.
 // All waits are bounded; on a timeout the kernel records it in the status word, drains the
 // copies and MMAs it issued, frees its TMEM and returns.
 #pragma once
@@ -28,11 +33,11 @@ namespace cobra {
 constexpr int kTcThreads = 192;
 constexpr uint64_t kTcWaitNs = 2000000000ull;  // 2 s
 constexpr int kTcEpiWarp0 = 2;
-constexpr int kTcTmemCols = 256;           // two accumulators of up to 128 columns
+constexpr int kTcStages = 3;               // X ring
+constexpr int kTcTmemCols = 256;           // two accumulators of 128 columns (tokens)
 constexpr int kTcXStageBytes = 2 * 16384;  // two 64-dim swizzle atoms of 128 rows
-constexpr int kTcCodeLd = 132;             // padded row stride of the code tile (bank spread)
 constexpr int kTcWBytes = 3 * 2 * 128 * 128;
-constexpr int kTcSmemBytes = 1024 + kTcWBytes + 2 * kTcXStageBytes + 128 * kTcCodeLd + 128 * 4 + 256;
+constexpr int kTcSmemBytes = 1024 + kTcWBytes + kTcStages * kTcXStageBytes + 256;
 
 struct TcArgs {
   const unsigned char* block;
@@ -75,18 +80,19 @@ __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t adesc, uin
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
-__device__ __forceinline__ void tc_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+// 32 consecutive TMEM columns of the warp's 32 lanes: v[j] = column (taddr + j) of this lane
+__device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+      "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
       : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
-        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),
+        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
       : "r"(taddr)
       : "memory");
 }
 __device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
@@ -106,19 +112,146 @@ __device__ __forceinline__ uint32_t umma_idesc_bf16(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
+// Epilogue state of one thread (one channel).
+struct TcEpi {
+  float inv_delta, cterm;  // u = y inv_delta + cterm, cterm = 2^{b-1} - (W^T mu)_i inv_delta
+  int cmax;
+};
+
+// Codes of the 32 tokens 32 c .. 32 c + 31 of this thread's channel into its sub-streams:
+// token t -> sub-stream t % 8, bits [(t / 8) B, (t / 8) B + B).
+template <int B, int C>
+__device__ __forceinline__ void tc_codes32(const uint32_t (&v)[32], const TcEpi& e, uint32_t (&sub)[8][(B + 1) / 2]) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const int t = 32 * C + j, sig = t & 7, pos = (t >> 3) * B;
+    int c = __float2int_rd(fmaf(__uint_as_float(v[j]), e.inv_delta, e.cterm));
+    c = min(max(c, 0), e.cmax);
+    const int k = pos >> 5, off = pos & 31;
+    sub[sig][k] |= (uint32_t)c << off;
+    if (off + B > 32) sub[sig][k + 1] |= (uint32_t)c >> (32 - off);
+  }
+}
+
+// Code row bytes [16 B i, 16 B (i + 1)) of channel i from the sub-streams (see the header).
+// K rows: word w of piece p = halfword w of sub-stream p of channel 2s (low) and of channel
+// 2s + 1 (high); lane pairs swap the four pieces the other one writes.  V rows: word w of piece
+// 4 (i % 2) + q = halfword w of sub-streams 2q (low) and 2q + 1 (high) of channel i.
+template <int B>
+__device__ __forceinline__ void tc_row_words(const uint32_t (&sub)[8][(B + 1) / 2], int side, int lane,
+                                             uint32_t (&words)[4 * B]) {
+  constexpr int NW = (B + 1) / 2;
+  const int par = lane & 1;
+  if (side == 0) {
+    uint32_t got[4][NW];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int k = 0; k < NW; ++k) {
+        const uint32_t send = par ? sub[j][k] : sub[4 + j][k];
+        got[j][k] = __shfl_xor_sync(0xffffffffu, send, 1);
+      }
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int w = 0; w < B; ++w) {
+        const uint32_t mine = par ? sub[4 + j][w >> 1] : sub[j][w >> 1];
+        const uint32_t lo = par ? got[j][w >> 1] : mine, hi = par ? mine : got[j][w >> 1];
+        words[j * B + w] = __byte_perm(lo, hi, (w & 1) ? 0x7632 : 0x5410);
+      }
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int w = 0; w < B; ++w)
+        words[q * B + w] = __byte_perm(sub[2 * q][w >> 1], sub[2 * q + 1][w >> 1], (w & 1) ? 0x7632 : 0x5410);
+  }
+}
+
+// The epilogue warps' loop over this CTA's tiles, for bit width B.
+template <int B>
+__device__ __forceinline__ void tc_epilogue(const TcArgs& a, const HeadEntry& he, const TcEpi& e, int chunk,
+                                            int my_tiles, int nrows, uint32_t tmem_q, uint32_t bar_acc_full,
+                                            uint32_t bar_acc_empty, int* fail) {
+  constexpr int NW = (B + 1) / 2;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int ch = 32 * (warp & 3) + lane;  // this thread's channel = its TMEM lane
+  const uint32_t rb = 16u * he.r * B;
+  for (int i = 0; i < my_tiles; ++i) {
+    const int acc = i & 1;
+    const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(bar_acc_full + 8u * acc, (i >> 1) & 1, kTcWaitNs));
+    if (!ok) {
+      if (lane == 0) {
+        atomicOr(&g_status, 1u);
+        *fail = 1;
+      }
+      break;
+    }
+    tc_fence_after();
+    uint32_t sub[8][NW];
+#pragma unroll
+    for (int s = 0; s < 8; ++s)
+#pragma unroll
+      for (int k = 0; k < NW; ++k) sub[s][k] = 0u;
+    const uint32_t tb = tmem_q + (uint32_t)(acc * 128);
+    {
+      uint32_t v[32];
+      tc_ld32(tb + 0, v);
+      tc_wait_ld();
+      tc_codes32<B, 0>(v, e, sub);
+      tc_ld32(tb + 32, v);
+      tc_wait_ld();
+      tc_codes32<B, 1>(v, e, sub);
+      tc_ld32(tb + 64, v);
+      tc_wait_ld();
+      tc_codes32<B, 2>(v, e, sub);
+      tc_ld32(tb + 96, v);
+      tc_wait_ld();
+      tc_codes32<B, 3>(v, e, sub);
+    }
+    // the accumulator can take the next tile's MMAs
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bar_acc_empty + 8u * acc);
+    const int tile = chunk + i * a.chunks;
+    const int seq = tile / nrows, row = tile % nrows;
+    const int nvalid = min(kRowTokens, a.n_tok - row * kRowTokens);
+    if (nvalid < kRowTokens) {
+      // tokens past the end are zero bits: sub-stream s keeps the codes rho < ceil((nvalid - s) / 8)
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        const int keep = max(0, min(16, (nvalid - s + 7) >> 3)) * B;
+#pragma unroll
+        for (int k = 0; k < NW; ++k) {
+          const int lo = 32 * k;
+          const uint32_t m = keep >= lo + 32 ? 0xffffffffu : (keep <= lo ? 0u : ((1u << (keep - lo)) - 1u));
+          sub[s][k] &= m;
+        }
+      }
+    }
+    uint32_t words[4 * B];
+    tc_row_words<B>(sub, a.side, lane, words);
+    if (ch < he.r) {
+      uint8_t* dst = a.cache + row_offset(he.cache_off, rb, seq, (a.t0 >> 7) + row, a.page_table, a.pages_per_seq,
+                                          a.rows_per_seq) + (size_t)ch * 16 * B;
+#pragma unroll
+      for (int k = 0; k < B; ++k)
+        reinterpret_cast<uint4*>(dst)[k] = make_uint4(words[4 * k], words[4 * k + 1], words[4 * k + 2], words[4 * k + 3]);
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kTcThreads, 1)
     compress_tc_kernel(const __grid_constant__ CUtensorMap xmap, TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);  // 1024-aligned for the swizzle
-  uint8_t* wsm = base;                                           // [split][atom][Npad rows][128 B]
-  uint8_t* xsm = wsm + kTcWBytes;                                // [stage][atom][128 rows][128 B]
-  uint8_t* codes = xsm + 2 * kTcXStageBytes;                     // [128 tokens][kTcCodeLd]
-  float* wmu_s = reinterpret_cast<float*>(codes + 128 * kTcCodeLd);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(wmu_s + 128);     // x_full[2] x_empty[2] acc_full[2] acc_empty[2] done
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 9);
-  int* counters = reinterpret_cast<int*>(tmem_holder + 1);       // [0] tiles issued by TMA, [1] consumed by MMA, [2] fail
-  int* epi_ok = counters + 4;                                    // one flag per epilogue warp
+  uint8_t* wsm = base;                                           // [split][atom][128 channels][128 B]
+  uint8_t* xsm = wsm + kTcWBytes;                                // [stage][atom][128 tokens][128 B]
+  // x_full[kTcStages] x_empty[kTcStages] acc_full[2] acc_empty[2] done
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xsm + kTcStages * kTcXStageBytes);
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * kTcStages + 5);
+  int* counters = reinterpret_cast<int*>(tmem_holder + 1);  // [0] tiles issued by TMA, [1] consumed by MMA, [2] fail
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int head_local = blockIdx.x / a.chunks, chunk = blockIdx.x % a.chunks;
@@ -129,28 +262,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int ntiles = a.n_seqs * nrows;
   if (r == 0 || chunk >= ntiles) return;
   const int my_tiles = (ntiles - chunk + a.chunks - 1) / a.chunks;
-  const int npad = (r + 15) & ~15;
   const int nsplit = b >= 6 ? 3 : 2;
   const float* pool = param_pool(a.block);
   const float* W = pool + he.w_off;
+  const uint32_t bar0 = smem_addr(bars);
+  auto bar = [&](int i) { return bar0 + 8u * i; };
+  const int XF = 0, XE = kTcStages, AF = 2 * kTcStages, AE = 2 * kTcStages + 2, DONE = 2 * kTcStages + 4;
 
-  // ---- setup: barriers, TMEM, split basis, W^T mu ----
+  // ---- setup: barriers, TMEM, split basis ----
   if (tid == 0) {
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(smem_addr(&bars[i]), 1);          // x_full: producer arrive + TMA bytes
-      mbar_init(smem_addr(&bars[2 + i]), 1);      // x_empty: MMA commit
-      mbar_init(smem_addr(&bars[4 + i]), 1);      // acc_full: MMA commit
-      mbar_init(smem_addr(&bars[6 + i]), 4);      // acc_empty: one arrive per epilogue warp
+    for (int i = 0; i < kTcStages; ++i) {
+      mbar_init(bar(XF + i), 1);  // producer arrive + TMA bytes
+      mbar_init(bar(XE + i), 1);  // MMA commit
     }
-    mbar_init(smem_addr(&bars[8]), 1);            // done: final MMA commit
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(AF + i), 1);  // MMA commit
+      mbar_init(bar(AE + i), 4);  // one arrive per epilogue warp
+    }
+    mbar_init(bar(DONE), 1);      // final MMA commit
     counters[0] = counters[1] = counters[2] = 0;
     fence_mbar_init();
   }
   if (warp == 1) tmem_alloc(smem_addr(tmem_holder), kTcTmemCols);
   // W split term sp of channel n, dims [64 atom, 64 atom + 64): 8 chunks of 16 bytes per row,
-  // chunk c stored at position c ^ (n & 7)
-  for (int idx = tid; idx < nsplit * 2 * npad * 8; idx += kTcThreads) {
-    const int c = idx & 7, n = (idx >> 3) % npad, atom = (idx / (8 * npad)) & 1, sp = idx / (16 * npad);
+  // chunk c stored at position c ^ (n & 7); channels n >= r are zero
+  for (int idx = tid; idx < nsplit * 2 * 128 * 8; idx += kTcThreads) {
+    const int c = idx & 7, n = (idx >> 3) & 127, atom = (idx >> 10) & 1, sp = idx >> 11;
     uint32_t packed[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -168,26 +305,23 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       }
       packed[e] = pack_bf16(v2[0], v2[1]);
     }
-    uint8_t* rowp = wsm + (size_t)sp * 2 * npad * 128 + (size_t)atom * npad * 128 + (size_t)n * 128;
+    uint8_t* rowp = wsm + (size_t)sp * 2 * 128 * 128 + (size_t)atom * 128 * 128 + (size_t)n * 128;
     *reinterpret_cast<uint4*>(rowp + ((c ^ (n & 7)) << 4)) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
   }
-  for (int i = tid; i < 128; i += kTcThreads) wmu_s[i] = i < r ? pool[he.wmu_off + i] : 0.f;
   // generic-proxy writes of the basis must be visible to the tensor cores (async proxy)
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
-  const uint32_t bar0 = smem_addr(bars);
-  auto bar = [&](int i) { return bar0 + 8u * i; };
 
   if (warp == 0) {
     // ---------------- TMA producer ----------------
     if (lane == 0) {
       int issued = 0;
       for (int i = 0; i < my_tiles; ++i) {
-        const int st = i & 1;
-        if (!mbar_wait_bounded(bar(2 + st), ((i >> 1) & 1) ^ 1, kTcWaitNs)) {
+        const int st = i % kTcStages, ph = (i / kTcStages) & 1;
+        if (!mbar_wait_bounded(bar(XE + st), ph ^ 1, kTcWaitNs)) {
           atomicOr(&g_status, 1u);
           counters[2] = 1;
           break;
@@ -200,25 +334,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         c[a.slot_tok] = row * kRowTokens;
         c[a.slot_seq] = seq;
         c[a.slot_layer] = layer;
-        mbar_arrive_expect_tx(bar(st), kTcXStageBytes);
+        mbar_arrive_expect_tx(bar(XF + st), kTcXStageBytes);
         const uint32_t dst = smem_addr(xsm + st * kTcXStageBytes);
-        tma_load_5d(dst, &xmap, c, bar(st));
+        tma_load_5d(dst, &xmap, c, bar(XF + st));
         c[0] = 64;
-        tma_load_5d(dst + 16384, &xmap, c, bar(st));
+        tma_load_5d(dst + 16384, &xmap, c, bar(XF + st));
         ++issued;
       }
       counters[0] = issued;
     }
   } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
+    // ---------------- MMA issuer: Y^T[128 channels][128 tokens] per tile ----------------
     if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(128, npad);
+      const uint32_t idesc = umma_idesc_bf16(128, 128);
       const uint32_t wbase = smem_addr(wsm), xbase = smem_addr(xsm);
       int consumed = 0;
       for (int i = 0; i < my_tiles; ++i) {
-        const int st = i & 1, acc = i & 1;
-        if (!mbar_wait_bounded(bar(st), (i >> 1) & 1, kTcWaitNs) ||
-            !mbar_wait_bounded(bar(6 + acc), ((i >> 1) & 1) ^ 1, kTcWaitNs)) {
+        const int st = i % kTcStages, acc = i & 1;
+        if (!mbar_wait_bounded(bar(XF + st), (i / kTcStages) & 1, kTcWaitNs) ||
+            !mbar_wait_bounded(bar(AE + acc), ((i >> 1) & 1) ^ 1, kTcWaitNs)) {
           atomicOr(&g_status, 1u);
           counters[2] = 1;
           break;
@@ -230,94 +364,41 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int sp = 0; sp < nsplit; ++sp)
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t aoff = (uint32_t)((kk >> 2) * 16384 + (kk & 3) * 32);
-            const uint32_t boff = (uint32_t)(sp * 2 * npad * 128 + (kk >> 2) * npad * 128 + (kk & 3) * 32);
-            tc_mma_bf16(d, umma_desc_sw128(xbase + st * kTcXStageBytes + aoff), umma_desc_sw128(wbase + boff), idesc,
-                        (sp > 0 || kk > 0) ? 1u : 0u);
+            const uint32_t koff = (uint32_t)((kk >> 2) * 16384 + (kk & 3) * 32);
+            tc_mma_bf16(d, umma_desc_sw128(wbase + sp * 2 * 16384 + koff),
+                        umma_desc_sw128(xbase + st * kTcXStageBytes + koff), idesc, (sp > 0 || kk > 0) ? 1u : 0u);
           }
-        tc_commit(bar(2 + st));   // X stage free once these MMAs completed
-        tc_commit(bar(4 + acc));  // accumulator ready
+        tc_commit(bar(XE + st));   // X stage free once these MMAs completed
+        tc_commit(bar(AF + acc));  // accumulator ready
       }
       counters[1] = consumed;
-      tc_commit(bar(8));  // completes when every MMA issued above has completed
-      if (!mbar_wait_bounded(bar(8), 0, kTcWaitNs)) atomicOr(&g_status, 1u);
+      tc_commit(bar(DONE));  // completes when every MMA issued above has completed
+      if (!mbar_wait_bounded(bar(DONE), 0, kTcWaitNs)) atomicOr(&g_status, 1u);
     }
   } else {
-    // ---------------- epilogue (warps 2..5) ----------------
-    const int q = warp & 3;               // TMEM lane quarter this warp may access
-    const int m = 32 * q + lane;          // token row of the tile
-    const int et = tid - kTcEpiWarp0 * 32;  // 0..127
-    const float inv_delta = he.inv_delta, half = (float)(1 << (b - 1));
-    const int cmax = (1 << b) - 1;
-    const uint32_t rb = 16u * r * b;
-    for (int i = 0; i < my_tiles; ++i) {
-      const int acc = i & 1;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(bar(4 + acc), (i >> 1) & 1, kTcWaitNs));
-      if (lane == 0) {
-        epi_ok[warp - kTcEpiWarp0] = ok ? 1 : 0;
-        if (!ok) {
-          atomicOr(&g_status, 1u);
-          counters[2] = 1;
-        }
-      }
-      // the four epilogue warps take the same decision from the same flags
-      named_bar_sync(1, 128);
-      const bool all_ok = epi_ok[0] && epi_ok[1] && epi_ok[2] && epi_ok[3];
-      named_bar_sync(1, 128);
-      if (!all_ok) break;
-      tc_fence_after();
-      const int tile = chunk + i * a.chunks;
-      const int seq = tile / nrows, row = tile % nrows;
-      const bool valid = row * kRowTokens + m < a.n_tok;
-      const uint32_t tbase = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(acc * 128);
-      for (int c0 = 0; c0 < npad; c0 += 16) {
-        uint32_t v[16];
-        tc_ld16(tbase + (uint32_t)c0, v);
-        tc_wait_ld();
-        uint32_t packed[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const int col = c0 + e;
-          const float y = __uint_as_float(v[e]) - wmu_s[col];
-          int code = (int)floorf(fmaf(y, inv_delta, half));
-          code = code < 0 ? 0 : (code > cmax ? cmax : code);
-          if (!valid || col >= r) code = 0;
-          packed[e >> 2] |= (uint32_t)code << (8 * (e & 3));
-        }
-        uint32_t* dstc = reinterpret_cast<uint32_t*>(codes + m * kTcCodeLd + c0);
-#pragma unroll
-        for (int e = 0; e < 4; ++e)
-          if (c0 + 4 * e < r) dstc[e] = packed[e];
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(bar(6 + acc));
-      named_bar_sync(1, 128);
-      uint8_t* dst = a.cache + row_offset(he.cache_off, rb, seq, (a.t0 >> 7) + row, a.page_table, a.pages_per_seq,
-                                          a.rows_per_seq);
-      const int npieces = 4 * r;
-      for (int idx = et; idx < npieces; idx += 128) {
-        const int s = idx >> 3, p = idx & 7;
-        uint32_t* out = reinterpret_cast<uint32_t*>(dst + s * 32 * b + p * 4 * b);
-        switch (b) {
-          case 1: pack_piece<1>(codes, kTcCodeLd, a.side, s, p, out); break;
-          case 2: pack_piece<2>(codes, kTcCodeLd, a.side, s, p, out); break;
-          case 3: pack_piece<3>(codes, kTcCodeLd, a.side, s, p, out); break;
-          case 4: pack_piece<4>(codes, kTcCodeLd, a.side, s, p, out); break;
-          case 5: pack_piece<5>(codes, kTcCodeLd, a.side, s, p, out); break;
-          case 6: pack_piece<6>(codes, kTcCodeLd, a.side, s, p, out); break;
-          case 7: pack_piece<7>(codes, kTcCodeLd, a.side, s, p, out); break;
-          default: pack_piece<8>(codes, kTcCodeLd, a.side, s, p, out); break;
-        }
-      }
-      named_bar_sync(1, 128);  // the code tile is rewritten by the next tile
+    // ---------------- epilogue (warps 2..5): one channel per thread ----------------
+    const int ch = 32 * (warp & 3) + lane;
+    TcEpi e;
+    e.inv_delta = he.inv_delta;
+    e.cterm = (float)(1 << (b - 1)) - (ch < r ? pool[he.wmu_off + ch] : 0.f) * he.inv_delta;
+    e.cmax = (1 << b) - 1;
+    const uint32_t tq = tmem + ((uint32_t)(32 * (warp & 3)) << 16);  // this warp's TMEM lane quarter
+    switch (b) {
+      case 1: tc_epilogue<1>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 2: tc_epilogue<2>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 3: tc_epilogue<3>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 4: tc_epilogue<4>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 5: tc_epilogue<5>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 6: tc_epilogue<6>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 7: tc_epilogue<7>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      default: tc_epilogue<8>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
     }
   }
   // ---- teardown: drain the TMA loads nobody consumed, then free TMEM ----
   __syncthreads();
   if (tid == 0) {
     for (int i = counters[1]; i < counters[0]; ++i)
-      if (!mbar_wait_bounded(bar(i & 1), (i >> 1) & 1, kTcWaitNs)) break;
+      if (!mbar_wait_bounded(bar(XF + i % kTcStages), (i / kTcStages) & 1, kTcWaitNs)) break;
   }
   tc_fence_before();
   __syncthreads();
