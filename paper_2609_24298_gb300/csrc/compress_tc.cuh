@@ -284,29 +284,48 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     fence_mbar_init();
   }
   if (warp == 1) tmem_alloc(smem_addr(tmem_holder), kTcTmemCols);
-  // W split term sp of channel n, dims [64 atom, 64 atom + 64): 8 chunks of 16 bytes per row,
-  // chunk c stored at position c ^ (n & 7); channels n >= r are zero
-  for (int idx = tid; idx < nsplit * 2 * 128 * 8; idx += kTcThreads) {
-    const int c = idx & 7, n = (idx >> 3) & 127, atom = (idx >> 10) & 1, sp = idx >> 11;
-    uint32_t packed[4];
+  // W split terms of channel n, dims [64 atom + 8 c, +8): one 16-byte chunk per term, stored at
+  // chunk position c ^ (n & 7) of the term's swizzled row; channels n >= r are zero.  Each
+  // chunk of W is loaded once (two 16-byte loads), four chunks per thread in flight together.
+  {
+    constexpr int kChunks = 2 * 128 * 8;  // (atom, channel, c)
+#pragma unroll 1
+    for (int base = 0; base < kChunks; base += 4 * kTcThreads) {
+      float4 wv[4][2];
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      float v2[2];
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int dim = 64 * atom + 8 * c + 2 * e + h;
-        float rem = n < r ? W[(size_t)n * kD + dim] : 0.f;
-        float part = 0.f;
-        for (int q = 0; q <= sp; ++q) {
-          part = __bfloat162float(__float2bfloat16_rn(rem));
-          rem -= part;
+      for (int u = 0; u < 4; ++u) {
+        const int idx = base + u * kTcThreads + tid;
+        const int c = idx & 7, n = (idx >> 3) & 127, atom = idx >> 10;
+        if (idx < kChunks && n < r) {
+          const float4* src = reinterpret_cast<const float4*>(W + (size_t)n * kD + 64 * atom + 8 * c);
+          wv[u][0] = src[0];
+          wv[u][1] = src[1];
+        } else {
+          wv[u][0] = wv[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
-        v2[h] = part;
       }
-      packed[e] = pack_bf16(v2[0], v2[1]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int idx = base + u * kTcThreads + tid;
+        if (idx >= kChunks) break;
+        const int c = idx & 7, n = (idx >> 3) & 127, atom = idx >> 10;
+        float rem[8] = {wv[u][0].x, wv[u][0].y, wv[u][0].z, wv[u][0].w, wv[u][1].x, wv[u][1].y, wv[u][1].z, wv[u][1].w};
+        for (int sp = 0; sp < nsplit; ++sp) {
+          uint32_t packed[4];
+#pragma unroll
+          for (int e2 = 0; e2 < 4; ++e2) {
+            const float p0 = __bfloat162float(__float2bfloat16_rn(rem[2 * e2]));
+            const float p1 = __bfloat162float(__float2bfloat16_rn(rem[2 * e2 + 1]));
+            rem[2 * e2] -= p0;
+            rem[2 * e2 + 1] -= p1;
+            packed[e2] = pack_bf16(p0, p1);
+          }
+          uint8_t* rowp = wsm + (size_t)sp * 2 * 128 * 128 + (size_t)atom * 128 * 128 + (size_t)n * 128;
+          *reinterpret_cast<uint4*>(rowp + ((c ^ (n & 7)) << 4)) =
+              make_uint4(packed[0], packed[1], packed[2], packed[3]);
+        }
+      }
     }
-    uint8_t* rowp = wsm + (size_t)sp * 2 * 128 * 128 + (size_t)atom * 128 * 128 + (size_t)n * 128;
-    *reinterpret_cast<uint4*>(rowp + ((c ^ (n & 7)) << 4)) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
   }
   // generic-proxy writes of the basis must be visible to the tensor cores (async proxy)
   fence_proxy_async_smem();
