@@ -235,23 +235,17 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
   for (int t = 0; t < 8; ++t)
 #pragma unroll
     for (int nt = 0; nt < NTK; ++nt) acc[t][nt][0] = acc[t][nt][1] = acc[t][nt][2] = acc[t][nt][3] = 0.f;
-  const int P = rk >> 1;
-  const int nfull = P >> 3, nk = (P + 7) >> 3;
-  // lane's pieces: strips 8 kappa + (lane & 3) and + 4, piece lane >> 2
+  const int nk = ((rk >> 1) + 7) >> 3;
+  // lane's pieces: strips 8 kappa + (lane & 3) and + 4, piece lane >> 2.  A partial last
+  // k-tile reads past the row (at most 7 strips, still inside the warp's shared memory): any
+  // word bits unpack to finite values, and channels past r multiply q~ = 0.
   const uint8_t* pa = stage + (lane & 3) * 32 * B + (lane >> 2) * 4 * B;
   const uint2* bq = bfrag + lane;
-  auto tile = [&](bool check, int kap) {
-    // channels past r (a partial last k-tile) multiply q~ = 0, so their operand values only
-    // need to be finite; the words are zeroed rather than read past the row
+#pragma unroll 1
+  for (int kap = 0; kap < nk; ++kap) {
     uint32_t wa[B], wb[B];
-    if (check) {
-      const int sA = 8 * kap + (lane & 3);
-      load_piece_or_zero<B>(pa, sA < P, wa);
-      load_piece_or_zero<B>(pa + 4 * 32 * B, sA + 4 < P, wb);
-    } else {
-      load_piece<B>(pa, wa);
-      load_piece<B>(pa + 4 * 32 * B, wb);
-    }
+    load_piece<B>(pa, wa);
+    load_piece<B>(pa + 4 * 32 * B, wb);
     uint2 bf[NTK];
 #pragma unroll
     for (int nt = 0; nt < NTK; ++nt) bf[nt] = bq[nt * 32];
@@ -264,10 +258,7 @@ __device__ __forceinline__ void k_row_scores(const uint8_t* stage, int rk, const
     }
     pa += 8 * 32 * B;
     bq += NTK * 32;
-  };
-#pragma unroll 1
-  for (int kap = 0; kap < nfull; ++kap) tile(false, kap);
-  if (nk > nfull) tile(true, nfull);
+  }
   // acc = Qsum + 2^(k-10) * sum_i q~_i code_i, Qsum = sum of the q~ fed to the MMA.  b >= 3
   // uses one window for every register, so Qsum shifts every token's score alike and softmax
   // ignores it; b = 1, 2 mix windows, so Qsum is removed before the per-token rescale:
