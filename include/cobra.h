@@ -181,10 +181,10 @@ cobra_status cobra_compress(const void* params, const cobra_compress_desc* desc,
 
 /* Append one token per sequence at device position pos[s] (Table alg:kvrobin step 7 applied
  * to the newly decoded token): x at x[l*sl + s*ss + h*sh + k] (x_stride_tok unused).  The
- * codes are written into the row bit by bit (other tokens' bits are kept); the row must hold
- * zero bits for this token beforehand (fresh caches are zero-filled; rows written by
- * cobra_compress have zero tails).  A position outside the cache's capacity is skipped and
- * flagged in the device status word (cobra_check returns COBRA_EINVAL). */
+ * token's code bits in its row are replaced (cleared, then set, with atomic word operations);
+ * the other tokens' bits are kept.  Appends of different positions of the same row may run
+ * concurrently.  A position outside the cache's capacity is skipped and flagged in the device
+ * status word (cobra_check returns COBRA_EINVAL). */
 cobra_status cobra_append(const void* params, const cobra_compress_desc* desc, const void* x, const int* pos,
                           uint8_t* cache, const int* page_table, void* stream);
 
@@ -282,6 +282,13 @@ cobra_status cobra_decode_attn_static(const void* params, const cobra_decode_des
  * bounded device wait expired since the last check, COBRA_EINVAL if a kernel skipped work
  * whose size did not fit its launch, COBRA_ECUDA on a CUDA error, else OK. */
 cobra_status cobra_check(void* stream);
+
+/* Self-test of the bounded-wait error path (the paper has no counterpart): one warp waits on a
+ * shared-memory barrier that nothing completes, gives up after limit_ns nanoseconds
+ * (0 < limit_ns <= 100 ms, else COBRA_EINVAL), records the expiry in the device status word
+ * exactly as the library's kernels do, and returns.  The next cobra_check(stream) then returns
+ * COBRA_ETIMEOUT and the context stays usable. */
+cobra_status cobra_selftest_wait_timeout(unsigned long long limit_ns, void* stream);
 
 #ifdef __cplusplus
 }

@@ -83,6 +83,7 @@ SIGNATURES = {
     "cobra_decode_attn_static": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), c_void_p, c_void_p, c_void_p, c_void_p,
                                          c_void_p, c_void_p]),
     "cobra_check": (c_int, [c_void_p]),
+    "cobra_selftest_wait_timeout": (c_int, [ctypes.c_ulonglong, c_void_p]),
 }
 
 _lib = None
@@ -326,3 +327,9 @@ def cobra_decode_attn_static(params, desc: DecodeDesc, q, cache, seq_lens, page_
 def cobra_check(stream=None) -> int:
     """Returns the status code (does not raise) so callers can test for COBRA_ETIMEOUT."""
     return lib().cobra_check(_stream(stream))
+
+
+def cobra_selftest_wait_timeout(limit_ns: int, stream=None):
+    """Launch the library's bounded-wait self-test (one warp waits on a barrier nothing
+    completes); the next cobra_check returns COBRA_ETIMEOUT."""
+    _chk("cobra_selftest_wait_timeout", lib().cobra_selftest_wait_timeout(int(limit_ns), _stream(stream)))

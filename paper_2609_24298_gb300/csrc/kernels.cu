@@ -464,6 +464,26 @@ extern "C" cobra_status cobra_decode_attn_static(const void* params, const cobra
   return launch_decode<8>(a, n_heads, (int)n_groups, kQproj | kScan | kCombine, s);
 }
 
+namespace {
+// One warp waits on a barrier that expects one arrival nobody makes.
+__global__ void selftest_wait_kernel(uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_addr(&bar), 1);
+    fence_mbar_init();
+  }
+  __syncwarp();
+  const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&bar), 0, limit_ns));
+  if (!ok && threadIdx.x == 0) atomicOr(&g_status, 1u);
+}
+}  // namespace
+
+extern "C" cobra_status cobra_selftest_wait_timeout(unsigned long long limit_ns, void* stream) {
+  if (limit_ns == 0 || limit_ns > 100000000ull) return COBRA_EINVAL;
+  selftest_wait_kernel<<<1, 32, 0, (cudaStream_t)stream>>>((uint64_t)limit_ns);
+  return launch_status();
+}
+
 extern "C" cobra_status cobra_check(void* stream) {
   if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return COBRA_ECUDA;
   unsigned int v = 0;

@@ -184,3 +184,10 @@ def test_binding_rejects_non_contiguous_buffers():
         cobra._ptr(x.t())
     with pytest.raises(ValueError):
         cobra._ptr(x[:, ::2])
+
+
+def test_selftest_wait_limits_checked_before_launch():
+    # limits outside (0, 100 ms] are refused on the host, before any device work
+    for bad in (0, 100_000_001):
+        with pytest.raises(Exception):
+            cobra.cobra_selftest_wait_timeout(bad)
