@@ -404,9 +404,8 @@ def run_cobra(args):
     if st != cobra.COBRA_OK:
         raise RuntimeError(f"device status {st} after warm-up")
 
-    # timed region: the whole steps, and the scan kernel alone (events on the launch stream)
+    # timed region: K whole steps, events only at its two ends (on the launch stream)
     K = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(K)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     if world > 1:
@@ -416,13 +415,20 @@ def run_cobra(args):
     time.sleep(0.3)
     t_start.record(stream)
     for k in range(K):
-        step(ev[k])
+        step()
     t_end.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
     if world > 1:
         dist.barrier()
     total_ms = t_start.elapsed_time(t_end)
+    # per-launch breakdown in a separate pass (events between the launches serialise them, so
+    # the timed region above has none)
+    KB = min(K, 200)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(KB)]
+    for k in range(KB):
+        step(ev[k])
+    torch.cuda.synchronize()
     stage_ms = {name: float(np.mean([e[i].elapsed_time(e[i + 1]) for e in ev])) for i, name in enumerate(stages)}
     scan_ms = stage_ms["scan"]
     if world > 1:

@@ -21,6 +21,13 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream serialisation may
+// start before the kernel ahead of it in the stream has finished; it calls grid_dep_wait()
+// before reading that kernel's results (a no-op for an ordinary launch).  grid_dep_launch()
+// lets the dependent kernel be scheduled once every CTA of this grid has called it or exited.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -72,8 +72,10 @@ __host__ __device__ constexpr size_t qproj_smem_bytes() {
   return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd);
 }
 constexpr int kWtChunk = 64;  // chunk weights held in shared memory per vector and round
+constexpr int kCombineVP = 16;  // query vectors per combine CTA (a head's sequences spread over CTAs)
+template <int VP>
 __host__ __device__ constexpr size_t combine_smem_bytes() {
-  return sizeof(float) * ((size_t)kD * kD + (size_t)kD * kZLd + kD + (size_t)kVecPass * kWtChunk);
+  return sizeof(float) * ((size_t)kD * kD + (size_t)kD * kZLd + kD + (size_t)VP * kWtChunk);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -662,6 +664,8 @@ __device__ __forceinline__ void scan_item(const DecodeArgs& a, ScanWarp& w, int 
 template <int G>
 __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs a) {
   extern __shared__ __align__(128) uint8_t smem[];
+  // the combine kernel may be scheduled as CTAs of this grid exit (it waits for the results)
+  grid_dep_launch();
   const int warp = threadIdx.x >> 5;
   ScanWarp w;
   w.lane = threadIdx.x & 31;
@@ -735,21 +739,25 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
 //   per query head: m* = max over chunks, l* = sum 2^(m - m*) l, zbar = Delta_V (sum 2^(m - m*)
 //   acc / l* - 2^{b-1} + 1/2), o = mu_V + W_V zbar (zeros for an empty sequence).
 // ---------------------------------------------------------------------------------------
-template <int G>
+// One CTA per (layer, kv head) and run of VP / G sequences (VP query vectors).
+template <int G, int VP>
 __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
-  constexpr int SPP = kVecPass / G;
+  constexpr int SPP = VP / G > 0 ? VP / G : 1;
+  static_assert(VP % 8 == 0 && VP <= kZLd, "combine pass width");
   extern __shared__ __align__(16) float csm[];
   float* Ws = csm;                  // [kD][kD]     W_V row i = channel i
   float* Zs = Ws + kD * kD;         // [kD][kZLd]   zbar of this pass, [channel][vector]
   float* mus = Zs + kD * kZLd;      // [kD]         mu_V
-  float* wts = mus + kD;            // [kVecPass][kWtChunk] normalised chunk weights
-  __shared__ float vinfo_m[kVecPass], vinfo_inv_l[kVecPass];
-  __shared__ int vinfo_first[kVecPass], vinfo_n[kVecPass], vinfo_g[kVecPass];
+  float* wts = mus + kD;            // [VP][kWtChunk] normalised chunk weights
+  __shared__ float vinfo_m[VP], vinfo_inv_l[VP];
+  __shared__ int vinfo_first[VP], vinfo_n[VP], vinfo_g[VP];
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
   const float* parts = reinterpret_cast<const float*>(a.ws + wh->part_off);
   const int S = wh->n_seqs;
-  const int* hg = reinterpret_cast<const int*>(a.ws + wh->hg_off) + (size_t)blockIdx.x * S;
+  const int nchunks = (S + SPP - 1) / SPP;
+  const int chunk = blockIdx.x % nchunks;
+  const int* hg = reinterpret_cast<const int*>(a.ws + wh->hg_off) + (size_t)(blockIdx.x / nchunks) * S;
   const WsGroup g0 = groups[hg[0]];
   const HeadEntry hv = head_table(a.block)[g0.v_head];
   const float* pool = param_pool(a.block);
@@ -758,15 +766,18 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   const float cen = rv > 0 ? (float)(1 << (hv.b - 1)) - 0.5f : 0.f;
   stage_basis(pool + hv.w_off, rv, kD, Ws);
   if (tid < kD) mus[tid] = pool[hv.mu_off + tid];
-  for (int s0 = 0; s0 < S; s0 += SPP) {
+  // everything above is independent of the scan; its partials are read only from here on
+  grid_dep_wait();
+  {
+    const int s0 = chunk * SPP;
     const int ns = min(SPP, S - s0), nv = ns * G;
-    __syncthreads();  // basis staged; the previous pass is done with Zs
+    __syncthreads();  // basis staged
     // (1) per vector (warp w: vectors w, w + 8, w + 16, w + 24): m* = max over the chunks and
     //     l* = sum 2^(m - m*) l, lanes over chunks, merged online (a chunk with no tokens has
     //     m = -inf and no value entries; its weight is zero).  The four vectors' loads are
     //     issued together.
     const int warp = tid >> 5, lane = tid & 31;
-    constexpr int NU = kVecPass / (kHeadThreads / 32);
+    constexpr int NU = VP / (kHeadThreads / 32);
     {
       const float* pg0[NU];
       int ni[NU];
@@ -830,9 +841,9 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
       const int i = tid & (kD - 1), par = tid >> 7;
       int kmax = 0;
       for (int v = 0; v < nv; ++v) kmax = max(kmax, vinfo_n[v]);
-      float acc[kVecPass / 2];
+      float acc[VP / 2];
 #pragma unroll
-      for (int q = 0; q < kVecPass / 2; ++q) acc[q] = 0.f;
+      for (int q = 0; q < VP / 2; ++q) acc[q] = 0.f;
       for (int k0 = 0; k0 < kmax; k0 += kWtChunk) {
         __syncthreads();  // the previous round's weights are consumed
         for (int idx = tid; idx < nv * kWtChunk; idx += kHeadThreads) {
@@ -848,7 +859,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
         if (i >= rv) continue;
         const int kr = min(kWtChunk, kmax - k0);
 #pragma unroll
-        for (int q0 = 0; q0 < kVecPass / 2; q0 += 4) {
+        for (int q0 = 0; q0 < VP / 2; q0 += 4) {
           if (2 * q0 + par >= nv) break;
           for (int kb = 0; kb < kr; kb += 8) {
             float x[4][8];
@@ -876,24 +887,28 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
         }
       }
 #pragma unroll
-      for (int q = 0; q < kVecPass / 2; ++q) {
+      for (int q = 0; q < VP / 2; ++q) {
         const int v = 2 * q + par;
         if (v >= nv) break;
         Zs[i * kZLd + v] = (i < rv && vinfo_first[v] >= 0) ? hv.delta * (acc[q] - cen) : 0.f;
       }
     }
     __syncthreads();
-    // thread: dims 4 (tid % 32) .. +3 for vectors 4 (tid / 32) .. +3
-    const int d0 = 4 * (tid & 31), v0 = 4 * (tid >> 5);
+    // thread: dims 4 (tid % 32) .. +3 for vectors VPW (tid / 32) .. +VPW-1
+    constexpr int VPW = VP / (kHeadThreads / 32);
+    const int d0 = 4 * (tid & 31), v0 = VPW * (tid >> 5);
     if (v0 < nv) {
       const float4 m4 = *reinterpret_cast<const float4*>(mus + d0);
-      float4 o[4] = {m4, m4, m4, m4};
+      float4 o[VPW];
+#pragma unroll
+      for (int v = 0; v < VPW; ++v) o[v] = m4;
       for (int i = 0; i < rv; ++i) {
         const float4 w = *reinterpret_cast<const float4*>(Ws + i * kD + d0);
-        const float4 z = *reinterpret_cast<const float4*>(Zs + i * kZLd + v0);
-        const float zz[4] = {z.x, z.y, z.z, z.w};
+        float zz[VPW];
 #pragma unroll
-        for (int v = 0; v < 4; ++v) {
+        for (int v = 0; v < VPW; ++v) zz[v] = Zs[i * kZLd + v0 + v];
+#pragma unroll
+        for (int v = 0; v < VPW; ++v) {
           o[v].x += w.x * zz[v];
           o[v].y += w.y * zz[v];
           o[v].z += w.z * zz[v];
@@ -901,7 +916,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
         }
       }
 #pragma unroll
-      for (int v = 0; v < 4; ++v) {
+      for (int v = 0; v < VPW; ++v) {
         const int vv = v0 + v;
         if (vv >= nv) break;
         const int seq = s0 + vv / G, g = vv % G;

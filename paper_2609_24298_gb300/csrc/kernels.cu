@@ -210,13 +210,13 @@ namespace {
 enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
 template <int G>
-cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_items, int stages, cudaStream_t s) {
+cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_items, int stages, cudaStream_t s) {
   static bool head_attr = false;
   if (!head_attr) {
     if (cudaFuncSetAttribute(qproj_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)qproj_smem_bytes()) !=
             cudaSuccess ||
-        cudaFuncSetAttribute(combine_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)combine_smem_bytes()) != cudaSuccess)
+        cudaFuncSetAttribute(combine_kernel<G, kCombineVP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)combine_smem_bytes<kCombineVP>()) != cudaSuccess)
       return COBRA_ECUDA;
     head_attr = true;
   }
@@ -245,7 +245,23 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_items, int st
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kCombine) {
-    combine_kernel<G><<<n_heads, kHeadThreads, combine_smem_bytes(), s>>>(a);
+    // one CTA per (layer, kv head) and run of kCombineVP / G sequences
+    constexpr int spp = kCombineVP / G > 0 ? kCombineVP / G : 1;
+    const long long grid = (long long)n_heads * ((n_seqs + spp - 1) / spp);
+    if (grid > 0x7fffffffLL) return COBRA_EINVAL;
+    // launched with programmatic stream serialisation: its prologue (basis staging) overlaps the
+    // scan's tail, and it waits for the scan before reading the partials
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kHeadThreads);
+    cfg.dynamicSmemBytes = combine_smem_bytes<kCombineVP>();
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, combine_kernel<G, kCombineVP>, a) != cudaSuccess) return COBRA_ECUDA;
     if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   }
   return COBRA_OK;
@@ -287,8 +303,8 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   cudaStream_t s = (cudaStream_t)stream;
   const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
   if (n_heads * d->n_seqs != info->n_groups) return COBRA_EINVAL;  // plan made for another descriptor
-  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, info->n_items, stages, s);
-  return launch_decode<8>(a, (int)n_heads, info->n_items, stages, s);
+  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s);
+  return launch_decode<8>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s);
 }
 }  // namespace
 
@@ -460,8 +476,8 @@ extern "C" cobra_status cobra_decode_attn_static(const void* params, const cobra
   a.one = kOneH2;
   a.ring_bytes = 2 * 16 * kD * 8;  // two rows of the largest head (r = 128, b = 8)
   const int n_heads = d->n_layers * d->n_kv_heads;
-  if (d->group == 4) return launch_decode<4>(a, n_heads, (int)n_groups, kQproj | kScan | kCombine, s);
-  return launch_decode<8>(a, n_heads, (int)n_groups, kQproj | kScan | kCombine, s);
+  if (d->group == 4) return launch_decode<4>(a, n_heads, d->n_seqs, (int)n_groups, kQproj | kScan | kCombine, s);
+  return launch_decode<8>(a, n_heads, d->n_seqs, (int)n_groups, kQproj | kScan | kCombine, s);
 }
 
 namespace {
