@@ -93,6 +93,22 @@ def hbm_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The largest of every rank's x (the slowest replica sets the time); x itself at N = 1."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def weak_scaling_gbs(bytes_per_step: int, steps: int, world: int, max_ms: float) -> float:
+    """Whole-job GB/s: every rank reads bytes_per_step per step; the job takes max_ms."""
+    return bytes_per_step * steps * world / (max_ms * 1e-3) / 1e9
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle-reason samples while the timed region runs."""
 
@@ -431,16 +447,13 @@ def run_cobra(args):
     torch.cuda.synchronize()
     stage_ms = {name: float(np.mean([e[i].elapsed_time(e[i + 1]) for e in ev])) for i, name in enumerate(stages)}
     scan_ms = stage_ms["scan"]
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, dev)
     st = cobra.cobra_check(stream)
     if st != cobra.COBRA_OK:
         raise RuntimeError(f"device status {st} after the timed region")
 
     bytes_step = pipeline.packed_bytes_read(wl)
-    value = bytes_step * K * world / (total_ms * 1e-3) / 1e9
+    value = weak_scaling_gbs(bytes_step, K, world, total_ms)
 
     # end to end through the public API: pinned host inputs in, host output out, every step
     hk = torch.empty_like(xk, device="cpu").pin_memory()
@@ -471,10 +484,7 @@ def run_cobra(args):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / Ke
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
     h2d = (xk.numel() + xv.numel() + q.numel()) * 2
     d2h = out.numel() * 4
 
@@ -498,7 +508,7 @@ def run_cobra(args):
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
             "compress": compress,
             "cpu_baseline": cpu,
-            "e2e": {"value": bytes_step * world / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s", "h2d_bytes_per_step": h2d,
+            "e2e": {"value": weak_scaling_gbs(bytes_step, 1, world, e2e_ms), "unit": "GB/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
             "stage_ms": stage_ms,
             "gpu_launches": launches_per_step * K,
