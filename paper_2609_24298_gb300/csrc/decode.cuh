@@ -75,7 +75,7 @@ constexpr int kWtChunk = 64;  // chunk weights held in shared memory per vector 
 constexpr int kCombineVP = 16;  // query vectors per combine CTA (a head's sequences spread over CTAs)
 template <int VP>
 __host__ __device__ constexpr size_t combine_smem_bytes() {
-  return sizeof(float) * ((size_t)kD * kD + (size_t)kD * kZLd + kD + (size_t)VP * kWtChunk);
+  return sizeof(float) * ((size_t)kD * kZLd + kD + (size_t)VP * kWtChunk);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -745,8 +745,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   constexpr int SPP = VP / G > 0 ? VP / G : 1;
   static_assert(VP % 8 == 0 && VP <= kZLd, "combine pass width");
   extern __shared__ __align__(16) float csm[];
-  float* Ws = csm;                  // [kD][kD]     W_V row i = channel i
-  float* Zs = Ws + kD * kD;         // [kD][kZLd]   zbar of this pass, [channel][vector]
+  float* Zs = csm;                  // [kD][kZLd]   zbar of this pass, [channel][vector]
   float* mus = Zs + kD * kZLd;      // [kD]         mu_V
   float* wts = mus + kD;            // [VP][kWtChunk] normalised chunk weights
   __shared__ float vinfo_m[VP], vinfo_inv_l[VP];
@@ -764,14 +763,15 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   const int rv = hv.r, layer = g0.layer, kv = g0.kv;
   const int tid = threadIdx.x;
   const float cen = rv > 0 ? (float)(1 << (hv.b - 1)) - 0.5f : 0.f;
-  stage_basis(pool + hv.w_off, rv, kD, Ws);
   if (tid < kD) mus[tid] = pool[hv.mu_off + tid];
+  // the rows of W_V are read through L1 in the back-projection (every warp reads the same rows)
+  const float4* W4 = reinterpret_cast<const float4*>(pool + hv.w_off);
   // everything above is independent of the scan; its partials are read only from here on
   grid_dep_wait();
   {
     const int s0 = chunk * SPP;
     const int ns = min(SPP, S - s0), nv = ns * G;
-    __syncthreads();  // basis staged
+    __syncthreads();  // mu_V staged
     // (1) per vector (warp w: vectors w, w + 8, w + 16, w + 24): m* = max over the chunks and
     //     l* = sum 2^(m - m*) l, lanes over chunks, merged online (a chunk with no tokens has
     //     m = -inf and no value entries; its weight is zero).  The four vectors' loads are
@@ -903,7 +903,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
 #pragma unroll
       for (int v = 0; v < VPW; ++v) o[v] = m4;
       for (int i = 0; i < rv; ++i) {
-        const float4 w = *reinterpret_cast<const float4*>(Ws + i * kD + d0);
+        const float4 w = __ldg(W4 + i * (kD / 4) + (d0 >> 2));
         float zz[VPW];
 #pragma unroll
         for (int v = 0; v < VPW; ++v) zz[v] = Zs[i * kZLd + v0 + v];
