@@ -25,8 +25,13 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
 // start before the kernel ahead of it in the stream has finished; it calls grid_dep_wait()
 // before reading that kernel's results (a no-op for an ordinary launch).  grid_dep_launch()
 // lets the dependent kernel be scheduled once every CTA of this grid has called it or exited.
+// Every kernel of the library is launched this way and calls grid_dep_wait() on every path
+// before it exits, so that the completion of a kernel implies that of all kernels before it
+// in the stream: a kernel only ever waits for its direct predecessor.
 __device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+// pull one 128-byte line into L2 (no register result, nothing to wait for)
+__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.global.L2 [%0];" ::"l"(p)); }
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -243,7 +248,8 @@ __device__ __forceinline__ void cp_async_wait_all() {
 // Rows [0, r) of a basis (fp32, 128 per row, 16-byte aligned) into shared memory with row
 // stride ld floats (a multiple of 4); rows [r, 128) are zeroed.  Every copy is issued before
 // any is waited for.  The caller synchronises the block before reading.
-__device__ __forceinline__ void stage_basis(const float* W, int r, int ld, float* dst) {
+// issues the copies only; the caller waits with cp_async_wait_all() before reading dst
+__device__ __forceinline__ void stage_basis_issue(const float* W, int r, int ld, float* dst) {
   for (int idx = threadIdx.x; idx < 128 * 32; idx += blockDim.x) {
     const int i = idx >> 5, c = idx & 31;
     float* d = dst + (size_t)i * ld + 4 * c;
@@ -252,6 +258,9 @@ __device__ __forceinline__ void stage_basis(const float* W, int r, int ld, float
     else
       *reinterpret_cast<float4*>(d) = make_float4(0.f, 0.f, 0.f, 0.f);
   }
+}
+__device__ __forceinline__ void stage_basis(const float* W, int r, int ld, float* dst) {
+  stage_basis_issue(W, r, ld, dst);
   cp_async_wait_all();
 }
 

@@ -79,12 +79,22 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* wmu = Ws + kD * kAppendWLd + (kAppendThreads / 32) * kD;  // W^T mu
   float* xs = Ws + kD * kAppendWLd + warp * kD;
+  grid_dep_launch();
   const int layer = blockIdx.x / a.n_kv, kv = blockIdx.x % a.n_kv;
   const HeadEntry he = head_table(a.block)[a.head0 + layer * a.layer_stride + kv];
   const int r = he.r, b = he.b;
-  if (r == 0) return;
+  if (r == 0) {
+    grid_dep_wait();
+    return;
+  }
   const float* pool = param_pool(a.block);
-  // the first sequence's token and position are loaded while the basis is staged
+  // the basis and W^T mu (r floats; the pool is padded to 32 floats, so whole 16-byte chunks
+  // stay in it) are parameters: their copies start before the wait for the kernel ahead
+  if (threadIdx.x < (r + 3) / 4) cp_async16(smem_addr(wmu + 4 * threadIdx.x), pool + he.wmu_off + 4 * threadIdx.x);
+  stage_basis_issue(pool + he.w_off, r, kAppendWLd, Ws);
+  // the tokens, positions and the cache may be produced or read by the kernels ahead
+  grid_dep_wait();
+  // the first sequence's token and position are loaded while the basis arrives
   __nv_bfloat16 xr[4];
   int p_next = 0;
   if (warp < a.n_seqs) {
@@ -93,9 +103,7 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) 
     for (int k = 0; k < 4; ++k) xr[k] = xp[lane + 32 * k];
     p_next = a.pos[warp];
   }
-  // W^T mu holds r floats (the pool is padded to 32 floats, so whole 16-byte chunks stay in it)
-  if (threadIdx.x < (r + 3) / 4) cp_async16(smem_addr(wmu + 4 * threadIdx.x), pool + he.wmu_off + 4 * threadIdx.x);
-  stage_basis(pool + he.w_off, r, kAppendWLd, Ws);
+  cp_async_wait_all();
   __syncthreads();
   const uint32_t rb = 16u * r * b;
   const float inv_delta = he.inv_delta, half = (float)(1 << (b - 1));

@@ -86,6 +86,7 @@ __host__ __device__ constexpr size_t combine_smem_bytes() {
 // ---------------------------------------------------------------------------------------
 template <int G>
 __global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
+  grid_dep_launch();
   constexpr int NTK = Heads<G>::NTK, SPP = kVecPass / G;
   extern __shared__ __align__(16) float qsm[];
   float* Ws = qsm;                  // [kD][kWLd]   W_K row i = channel i
@@ -101,7 +102,11 @@ __global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
   const int r = hk.r, layer = g0.layer, kv = g0.kv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float scale = hk.delta * 0.088388347648318440f * 1.4426950408889634f;  // Delta/sqrt(128)*log2(e)
-  stage_basis(pool + hk.w_off, r, kWLd, Ws);
+  // the basis is a parameter: its copy overlaps the end of the kernel ahead; the queries and
+  // the q~ blocks of the workspace are touched only after the wait
+  stage_basis_issue(pool + hk.w_off, r, kWLd, Ws);
+  grid_dep_wait();
+  cp_async_wait_all();
   for (int s0 = 0; s0 < S; s0 += SPP) {
     const int ns = min(SPP, S - s0), nv = ns * G;
     __syncthreads();  // basis staged; the previous pass is done with Qs and Os
@@ -686,6 +691,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
     fence_mbar_init();
   }
   __syncwarp();
+  // the q~ blocks come from the query projection ahead, the cache from the appends before it
+  grid_dep_wait();
 
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
@@ -732,6 +739,16 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
       if (++w.wait_stage == w.nstage) w.wait_stage = 0;
     }
   }
+  // the last CTA to run out of items puts the work counter back to 0 for the next launch:
+  // by then every warp of the grid has taken its final (empty) index
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned int* done = const_cast<unsigned int*>(&wh->done_ctas);
+    if (atomicAdd(done, 1u) == gridDim.x - 1) {
+      atomicExch(next_item, 0u);
+      atomicExch(done, 0u);
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------------------
@@ -764,8 +781,12 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   const int tid = threadIdx.x;
   const float cen = rv > 0 ? (float)(1 << (hv.b - 1)) - 0.5f : 0.f;
   if (tid < kD) mus[tid] = pool[hv.mu_off + tid];
-  // the rows of W_V are read through L1 in the back-projection (every warp reads the same rows)
+  // the rows of W_V are read through L1 in the back-projection (every warp reads the same rows);
+  // they are pulled into L2 here, while the scan ahead of this kernel is still finishing
   const float4* W4 = reinterpret_cast<const float4*>(pool + hv.w_off);
+  for (int idx = tid; idx < rv * (kD / 32); idx += kHeadThreads) prefetch_l2(pool + hv.w_off + 32 * idx);
+  // the appends of the next step may start their parameter staging meanwhile
+  grid_dep_launch();
   // everything above is independent of the scan; its partials are read only from here on
   grid_dep_wait();
   {
@@ -902,8 +923,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
       float4 o[VPW];
 #pragma unroll
       for (int v = 0; v < VPW; ++v) o[v] = m4;
-      for (int i = 0; i < rv; ++i) {
-        const float4 w = __ldg(W4 + i * (kD / 4) + (d0 >> 2));
+      auto accum = [&](const float4& w, int i) {
         float zz[VPW];
 #pragma unroll
         for (int v = 0; v < VPW; ++v) zz[v] = Zs[i * kZLd + v0 + v];
@@ -914,7 +934,17 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
           o[v].z += w.z * zz[v];
           o[v].w += w.w * zz[v];
         }
+      };
+      // rows in blocks of 8 whose loads are all issued before the first is used
+      int i = 0;
+      for (; i + 8 <= rv; i += 8) {
+        float4 w[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) w[u] = __ldg(W4 + (i + u) * (kD / 4) + (d0 >> 2));
+#pragma unroll
+        for (int u = 0; u < 8; ++u) accum(w[u], i + u);
       }
+      for (; i < rv; ++i) accum(__ldg(W4 + i * (kD / 4) + (d0 >> 2)), i);
 #pragma unroll
       for (int v = 0; v < VPW; ++v) {
         const int vv = v0 + v;

@@ -54,8 +54,9 @@ struct WsHeader {
   int32_t max_row_bytes;  // largest K or V code row among the planned heads
   int32_t reserved0;
   uint64_t hg_off;        // int32 [n_layers * n_kv][n_seqs]: group index of (head, seq)
-  int32_t reserved[7];
-  uint32_t next_item;     // scan work counter: zeroed on the stream before every scan launch
+  int32_t reserved[6];
+  uint32_t done_ctas;     // scan CTAs that have finished taking items in the running launch
+  uint32_t next_item;     // scan work counter: 0 between launches (the scan's last CTA resets it)
 };
 static_assert(sizeof(WsHeader) == 128, "ws header size");
 

@@ -168,6 +168,27 @@ extern "C" cobra_status cobra_compress(const void* params, const cobra_compress_
   return launch_status();
 }
 
+namespace {
+// Launch with programmatic stream serialisation: the kernel may become resident while the one
+// ahead of it in the stream finishes; it waits for that kernel (grid_dep_wait) before touching
+// anything the kernel ahead may produce or read.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), unsigned grid, unsigned block, size_t smem, cudaStream_t s,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+}  // namespace
+
 extern "C" cobra_status cobra_append(const void* params, const cobra_compress_desc* d, const void* x, const int* pos,
                                      uint8_t* cache, const int* page_table, void* stream) {
   cobra_status st = check_compress_desc(d);
@@ -201,7 +222,9 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
       return COBRA_ECUDA;
     attr = true;
   }
-  append_kernel<<<(unsigned)grid, kAppendThreads, append_smem_bytes(), (cudaStream_t)stream>>>(a);
+  if (launch_pdl(append_kernel, (unsigned)grid, kAppendThreads, append_smem_bytes(), (cudaStream_t)stream, a) !=
+      cudaSuccess)
+    return COBRA_ECUDA;
   return launch_status();
 }
 
@@ -210,7 +233,8 @@ namespace {
 enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
 template <int G>
-cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_items, int stages, cudaStream_t s) {
+cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_items, int stages, cudaStream_t s,
+                           bool after_plan_kernel = false) {
   static bool head_attr = false;
   if (!head_attr) {
     if (cudaFuncSetAttribute(qproj_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)qproj_smem_bytes()) !=
@@ -221,8 +245,14 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
     head_attr = true;
   }
   if (stages & kQproj) {
-    qproj_kernel<G><<<n_heads, kHeadThreads, qproj_smem_bytes(), s>>>(a);
-    if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
+    // the query projection reads the plan before its wait; right after the plan kernel it is
+    // launched in plain stream order
+    if (after_plan_kernel) {
+      qproj_kernel<G><<<n_heads, kHeadThreads, qproj_smem_bytes(), s>>>(a);
+      if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
+    } else if (launch_pdl(qproj_kernel<G>, (unsigned)n_heads, kHeadThreads, qproj_smem_bytes(), s, a) != cudaSuccess) {
+      return COBRA_ECUDA;
+    }
   }
   if (stages & kScan) {
     const size_t smem =
@@ -239,30 +269,18 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
     per_sm = std::max(per_sm, 1);
     const int want = (n_items + kDecodeWarps - 1) / kDecodeWarps;
     const int grid = std::max(1, std::min(want, per_sm * sm_count()));
-    if (cudaMemsetAsync(a.ws + offsetof(WsHeader, next_item), 0, sizeof(uint32_t), s) != cudaSuccess)
-      return COBRA_ECUDA;
-    decode_kernel<G><<<grid, kDecodeWarps * 32, smem, s>>>(a);
-    if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
+    // the work counter is 0 here: the plan writes it so, and every scan's last CTA resets it
+    if (launch_pdl(decode_kernel<G>, (unsigned)grid, kDecodeWarps * 32, smem, s, a) != cudaSuccess) return COBRA_ECUDA;
   }
   if (stages & kCombine) {
     // one CTA per (layer, kv head) and run of kCombineVP / G sequences
     constexpr int spp = kCombineVP / G > 0 ? kCombineVP / G : 1;
     const long long grid = (long long)n_heads * ((n_seqs + spp - 1) / spp);
     if (grid > 0x7fffffffLL) return COBRA_EINVAL;
-    // launched with programmatic stream serialisation: its prologue (basis staging) overlaps the
-    // scan's tail, and it waits for the scan before reading the partials
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)grid);
-    cfg.blockDim = dim3(kHeadThreads);
-    cfg.dynamicSmemBytes = combine_smem_bytes<kCombineVP>();
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, combine_kernel<G, kCombineVP>, a) != cudaSuccess) return COBRA_ECUDA;
-    if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
+    // its prologue (mu_V, the L2 prefetch of W_V) overlaps the scan's tail
+    if (launch_pdl(combine_kernel<G, kCombineVP>, (unsigned)grid, kHeadThreads, combine_smem_bytes<kCombineVP>(), s,
+                   a) != cudaSuccess)
+      return COBRA_ECUDA;
   }
   return COBRA_OK;
 }
@@ -476,8 +494,8 @@ extern "C" cobra_status cobra_decode_attn_static(const void* params, const cobra
   a.one = kOneH2;
   a.ring_bytes = 2 * 16 * kD * 8;  // two rows of the largest head (r = 128, b = 8)
   const int n_heads = d->n_layers * d->n_kv_heads;
-  if (d->group == 4) return launch_decode<4>(a, n_heads, d->n_seqs, (int)n_groups, kQproj | kScan | kCombine, s);
-  return launch_decode<8>(a, n_heads, d->n_seqs, (int)n_groups, kQproj | kScan | kCombine, s);
+  if (d->group == 4) return launch_decode<4>(a, n_heads, d->n_seqs, (int)n_groups, kQproj | kScan | kCombine, s, true);
+  return launch_decode<8>(a, n_heads, d->n_seqs, (int)n_groups, kQproj | kScan | kCombine, s, true);
 }
 
 namespace {
