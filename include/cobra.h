@@ -222,12 +222,23 @@ typedef struct {
   int reserved;
 } cobra_decode_info;
 
-/* Write the work plan (token chunks sized by bytes, per (seq, layer, kv-head)) into the
+/* Write the work plan (token chunks of whole code rows per (seq, layer, kv-head), in the order
+ * the scan takes them; the chunks shrink towards the end of the order, so that the scan's warps
+ * finish close together) into the
  * device workspace (one cudaMemcpyAsync on `stream`; the call synchronises the stream
  * before returning) and describe it in *info.  The plan stays valid for any
  * seq_lens[s] <= seq_cap[s] and for any parameter block whose heads have the same (r, b). */
 cobra_status cobra_decode_plan(const cobra_decode_desc* desc, const int* head_r, const int* head_b, const int* seq_cap,
                                void* workspace, size_t ws_bytes, cobra_decode_info* info, void* stream);
+
+/* The same plan written to host memory instead: `image` receives the first *written bytes of a
+ * planned workspace (header, chunk groups, chunks in the order the scan takes them, head-group
+ * table); copying them to the start of a workspace of cobra_decode_workspace_size bytes plans
+ * it.  With image == NULL (or too small) only *written is set, and the call returns
+ * COBRA_EINVAL (COBRA_ESPACE).  Needs no device. */
+cobra_status cobra_decode_plan_host(const cobra_decode_desc* desc, const int* head_r, const int* head_b,
+                                    const int* seq_cap, void* image, size_t image_bytes, size_t* written,
+                                    cobra_decode_info* info);
 
 /* Run decode attention with a planned workspace.  q: device bf16; seq_lens: device int32
  * [n_seqs] (0 gives an all-zero output for that sequence); out: device fp32.  Three

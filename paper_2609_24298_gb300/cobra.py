@@ -72,6 +72,8 @@ SIGNATURES = {
     "cobra_decode_workspace_size": (c_int, [ctypes.POINTER(DecodeDesc), P_int, P_int, P_int, P_size]),
     "cobra_decode_plan": (c_int, [ctypes.POINTER(DecodeDesc), P_int, P_int, P_int, c_void_p, c_size_t,
                                   ctypes.POINTER(DecodeInfo), c_void_p]),
+    "cobra_decode_plan_host": (c_int, [ctypes.POINTER(DecodeDesc), P_int, P_int, P_int, c_void_p, c_size_t, P_size,
+                                       ctypes.POINTER(DecodeInfo)]),
     "cobra_decode_attn": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo), c_void_p,
                                   c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t, c_void_p]),
     "cobra_decode_qproj": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo), c_void_p,
@@ -288,6 +290,23 @@ def cobra_decode_plan(desc: DecodeDesc, head_r, head_b, seq_cap, workspace, ws_b
                                  _stream(stream))
     _chk("cobra_decode_plan", st)
     return info
+
+
+def cobra_decode_plan_host(desc: DecodeDesc, head_r, head_b, seq_cap):
+    """The plan as host bytes (the first bytes of a planned workspace) and its DecodeInfo."""
+    hr, hrp = _np(head_r, np.int32, c_int)
+    hb, hbp = _np(head_b, np.int32, c_int)
+    sc, scp = _np(seq_cap, np.int32, c_int)
+    n = c_size_t(0)
+    info = DecodeInfo()
+    st = lib().cobra_decode_plan_host(ctypes.byref(desc), hrp, hbp, scp, None, 0, ctypes.byref(n), ctypes.byref(info))
+    if st != COBRA_EINVAL or n.value == 0:
+        _chk("cobra_decode_plan_host", st)
+    img = np.zeros(n.value, np.uint8)
+    st = lib().cobra_decode_plan_host(ctypes.byref(desc), hrp, hbp, scp, img.ctypes.data, img.size, ctypes.byref(n),
+                                      ctypes.byref(info))
+    _chk("cobra_decode_plan_host", st)
+    return img, info
 
 
 def cobra_decode_attn(params, desc: DecodeDesc, info: DecodeInfo, q, cache, seq_lens, page_table, out, workspace,

@@ -474,7 +474,7 @@ __device__ __forceinline__ void scan_item(const DecodeArgs& a, ScanWarp& w, int 
   const int T = a.seq_lens[gr.seq];
   const int rows_valid = (T + kRowTokens - 1) / kRowTokens;
   const int row0 = it.row_begin, row1 = min(it.row_end, rows_valid);
-  float* part = parts + (size_t)item * pstride;
+  float* part = parts + (size_t)it.slot * pstride;
   const uint32_t rbk = kr > 0 ? 16u * kr * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
   // one stage = this item's K row + V row (every load of the previous item has been
   // consumed, so the whole ring is free)

@@ -667,11 +667,20 @@ extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, 
 }
 
 // ----------------------------------------------------------------------------------------
-// Decode work plan: per (seq, layer, kv-head) group, token chunks of whole code rows sized so
-// that each chunk reads about kItemBytes of packed K+V codes.
+// Decode work plan: per (seq, layer, kv-head) group, token chunks of whole code rows.  The
+// scan's warps take the chunks in plan order, and the chunk sizes shrink towards the end of
+// the list (guided self-scheduling): a chunk holds about the packed K+V bytes still ahead of it
+// divided by kGuide x kScanWarps, clamped to [kItemMin, kItemMax], and no group is cut into
+// more than about kMaxChunks chunks (the combine merges a group's chunks).  Most of the cache
+// goes in large chunks (little per-chunk setup), and the warps that drain the queue finish
+// within one short chunk of one another.  Groups are ordered by code variant (b_K, b_V), then
+// (r_K, r_V), so that the warps working at the same time run the same code.
 // ----------------------------------------------------------------------------------------
 namespace {
-constexpr long long kItemBytes = 64 * 1024;
+constexpr long long kItemMin = 16 * 1024, kItemMax = 256 * 1024;
+constexpr long long kScanWarps = 152 * 16;  // resident scan warps: 152 SMs x 4 CTAs x 4 warps
+constexpr long long kGuide = 2;
+constexpr long long kMaxChunks = 32;
 
 cobra_status check_decode_desc(const cobra_decode_desc* d) {
   if (!d) return COBRA_EINVAL;
@@ -698,8 +707,6 @@ cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int*
     if (!d->pages_per_seq && rows > d->rows_per_seq) return COBRA_EINVAL;
     if (d->pages_per_seq && rows > 2LL * d->pages_per_seq) return COBRA_EINVAL;
   }
-  // groups ordered by (b_K, b_V, r_K, r_V, seq, layer, kv) so that the warps working on
-  // neighbouring chunks at the same time run the same code variant
   struct Key {
     int bk, bv, rk, rv, s, l, h;
   };
@@ -708,7 +715,10 @@ cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int*
     for (int l = 0; l < d->n_layers; ++l)
       for (int h = 0; h < d->n_kv_heads; ++h) {
         const int hk = d->k_head0 + l * d->layer_stride + h, hv = d->v_head0 + l * d->layer_stride + h;
-        keys.push_back({head_r[hk] ? head_b[hk] : 0, head_r[hv] ? head_b[hv] : 0, head_r[hk], head_r[hv], s, l, h});
+        const int rk = head_r[hk], rv = head_r[hv], bk = rk ? head_b[hk] : 0, bv = rv ? head_b[hv] : 0;
+        if (rk < 0 || rk > 128 || (rk & 1) || rv < 0 || rv > 128 || (rv & 1) || bk < 0 || bk > 8 || bv < 0 || bv > 8)
+          return COBRA_EINVAL;
+        keys.push_back({bk, bv, rk, rv, s, l, h});
       }
   std::stable_sort(keys.begin(), keys.end(), [](const Key& x, const Key& y) {
     if (x.bk != y.bk) return x.bk < y.bk;
@@ -716,29 +726,33 @@ cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int*
     if (x.rk != y.rk) return x.rk < y.rk;
     return x.rv < y.rv;
   });
+  auto pair_bytes = [](const Key& k) {
+    return (long long)cobra_row_bytes(k.rk, k.bk) + (long long)cobra_row_bytes(k.rv, k.bv);
+  };
+  long long remaining = 0;  // packed K+V bytes not yet in a chunk
+  for (const Key& k : keys) remaining += (long long)(seq_cap[k.s] + 127) / 128 * pair_bytes(k);
   for (const Key& key : keys) {
-      {
-        const int s = key.s, l = key.l, h = key.h;
-        const int hk = d->k_head0 + l * d->layer_stride + h, hv = d->v_head0 + l * d->layer_stride + h;
-        const int rk = head_r[hk], bk = head_r[hk] ? head_b[hk] : 0, rv = head_r[hv], bv = head_r[hv] ? head_b[hv] : 0;
-        if (rk < 0 || rk > 128 || (rk & 1) || rv < 0 || rv > 128 || (rv & 1) || bk < 0 || bk > 8 || bv < 0 || bv > 8)
-          return COBRA_EINVAL;
-        p.max_rv = std::max(p.max_rv, rv);
-        p.max_row_bytes = std::max(p.max_row_bytes, (int)std::max(cobra_row_bytes(rk, bk), cobra_row_bytes(rv, bv)));
-        const long long rows = (seq_cap[s] + 127) / 128;
-        const long long row_bytes = (long long)cobra_row_bytes(rk, bk) + (long long)cobra_row_bytes(rv, bv);
-        long long n_items = rows == 0 ? 1 : std::max(1LL, (rows * row_bytes + kItemBytes - 1) / kItemBytes);
-        n_items = std::min(n_items, std::max(rows, 1LL));
-        const long long per = rows == 0 ? 0 : (rows + n_items - 1) / n_items;
-        cobra::WsGroup g{s, l, h, (int)p.items.size(), 0, hk, hv, 0};
-        for (long long k = 0; k < n_items; ++k) {
-          const long long r0 = std::min(rows, k * per), r1 = std::min(rows, (k + 1) * per);
-          if (r1 <= r0 && k > 0) break;
-          p.items.push_back({(int)p.groups.size(), (int)r0, (int)r1, 0});
-          g.n_items++;
-        }
-        p.groups.push_back(g);
-      }
+    const int hk = d->k_head0 + key.l * d->layer_stride + key.h, hv = d->v_head0 + key.l * d->layer_stride + key.h;
+    p.max_rv = std::max(p.max_rv, key.rv);
+    p.max_row_bytes =
+        std::max(p.max_row_bytes, (int)std::max(cobra_row_bytes(key.rk, key.bk), cobra_row_bytes(key.rv, key.bv)));
+    const long long rows = (seq_cap[key.s] + 127) / 128, rb = pair_bytes(key);
+    cobra::WsGroup g{key.s, key.l, key.h, (int)p.items.size(), 0, hk, hv, 0};
+    if (rows == 0 || rb == 0) {  // one (empty or code-less) chunk
+      p.items.push_back({(int)p.groups.size(), 0, (int)rows, (int)p.items.size()});
+      g.n_items = 1;
+    }
+    const long long min_rows = (rows + kMaxChunks - 1) / kMaxChunks;
+    for (long long r0 = 0; r0 < rows && rb > 0;) {
+      const long long target = std::min(kItemMax, std::max(kItemMin, remaining / (kGuide * kScanWarps)));
+      long long n = std::max(min_rows, std::max(1LL, (target + rb / 2) / rb));
+      if (rows - r0 - n < (n + 1) / 2) n = rows - r0;  // no short remainder chunk
+      p.items.push_back({(int)p.groups.size(), (int)r0, (int)(r0 + n), (int)p.items.size()});
+      g.n_items++;
+      r0 += n;
+      remaining -= n * rb;
+    }
+    p.groups.push_back(g);
   }
   return COBRA_OK;
 }
@@ -784,20 +798,17 @@ extern "C" cobra_status cobra_decode_workspace_size(const cobra_decode_desc* des
   return COBRA_OK;
 }
 
-extern "C" cobra_status cobra_decode_plan(const cobra_decode_desc* desc, const int* head_r, const int* head_b,
-                                          const int* seq_cap, void* workspace, size_t ws_bytes, cobra_decode_info* info,
-                                          void* stream) {
+namespace {
+// header + groups + items + head-group table of the workspace, as a host image
+cobra_status plan_image(const cobra_decode_desc* desc, const int* head_r, const int* head_b, const int* seq_cap,
+                        std::vector<unsigned char>& img, size_t* ws_need, cobra_decode_info* info) {
   Plan p;
   cobra_status st = make_plan(desc, head_r, head_b, seq_cap, p);
   if (st != COBRA_OK) return st;
-  if (!workspace || !info) return COBRA_EINVAL;
-  if (((uintptr_t)workspace) & 255) return COBRA_EALIGN;
   cobra::WsHeader h;
-  size_t need;
-  ws_layout(desc, p, h, need);
-  if (ws_bytes < need) return COBRA_ESPACE;
-  const size_t head_bytes = h.qt_off;  // header + groups + items + head-group table
-  std::vector<unsigned char> img(head_bytes, 0);
+  ws_layout(desc, p, h, *ws_need);
+  const size_t head_bytes = h.qt_off;
+  img.assign(head_bytes, 0);
   std::memcpy(img.data(), &h, sizeof(h));
   std::memcpy(img.data() + h.groups_off, p.groups.data(), sizeof(cobra::WsGroup) * p.groups.size());
   std::memcpy(img.data() + h.items_off, p.items.data(), sizeof(cobra::WsItem) * p.items.size());
@@ -806,12 +817,45 @@ extern "C" cobra_status cobra_decode_plan(const cobra_decode_desc* desc, const i
     const cobra::WsGroup& gr = p.groups[g];
     hg[((size_t)gr.layer * desc->n_kv_heads + gr.kv) * desc->n_seqs + gr.seq] = (int32_t)g;
   }
-  cudaStream_t s = (cudaStream_t)stream;
-  if (cudaMemcpyAsync(workspace, img.data(), head_bytes, cudaMemcpyHostToDevice, s) != cudaSuccess) return COBRA_ECUDA;
-  if (cudaStreamSynchronize(s) != cudaSuccess) return COBRA_ECUDA;
   info->n_groups = h.n_groups;
   info->n_items = h.n_items;
   info->max_row_bytes = h.max_row_bytes;
   info->reserved = 0;
+  return COBRA_OK;
+}
+}  // namespace
+
+extern "C" cobra_status cobra_decode_plan_host(const cobra_decode_desc* desc, const int* head_r, const int* head_b,
+                                               const int* seq_cap, void* image, size_t image_bytes, size_t* written,
+                                               cobra_decode_info* info) {
+  if (!written || !info) return COBRA_EINVAL;
+  std::vector<unsigned char> img;
+  size_t need = 0;
+  cobra_decode_info inf{};
+  cobra_status st = plan_image(desc, head_r, head_b, seq_cap, img, &need, &inf);
+  if (st != COBRA_OK) return st;
+  *written = img.size();
+  if (!image) return COBRA_EINVAL;
+  if (image_bytes < img.size()) return COBRA_ESPACE;
+  std::memcpy(image, img.data(), img.size());
+  *info = inf;
+  return COBRA_OK;
+}
+
+extern "C" cobra_status cobra_decode_plan(const cobra_decode_desc* desc, const int* head_r, const int* head_b,
+                                          const int* seq_cap, void* workspace, size_t ws_bytes, cobra_decode_info* info,
+                                          void* stream) {
+  if (!workspace || !info) return COBRA_EINVAL;
+  if (((uintptr_t)workspace) & 255) return COBRA_EALIGN;
+  std::vector<unsigned char> img;
+  size_t need = 0;
+  cobra_decode_info inf{};
+  cobra_status st = plan_image(desc, head_r, head_b, seq_cap, img, &need, &inf);
+  if (st != COBRA_OK) return st;
+  if (ws_bytes < need) return COBRA_ESPACE;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (cudaMemcpyAsync(workspace, img.data(), img.size(), cudaMemcpyHostToDevice, s) != cudaSuccess) return COBRA_ECUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return COBRA_ECUDA;
+  *info = inf;
   return COBRA_OK;
 }

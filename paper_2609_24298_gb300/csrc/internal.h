@@ -60,12 +60,14 @@ struct WsHeader {
 };
 static_assert(sizeof(WsHeader) == 128, "ws header size");
 
+// A group's chunks write their partials to slots first_item .. first_item + n_items - 1.
 struct WsGroup {
   int32_t seq, layer, kv, first_item;
   int32_t n_items, k_head, v_head, reserved;
 };
+// Work items in the order the scan takes them; slot is the partial the chunk writes.
 struct WsItem {
-  int32_t group, row_begin, row_end, reserved;
+  int32_t group, row_begin, row_end, slot;
 };
 
 // q~ block per group: Qsum[8] (fp32, sum of the fp16 hi+lo values per query head),

@@ -424,7 +424,7 @@ __global__ void static_plan_kernel(unsigned char* ws, const unsigned char* block
     const int h = g % d.n_kv_heads, l = (g / d.n_kv_heads) % d.n_layers, s = g / (d.n_kv_heads * d.n_layers);
     const int hk = d.k_head0 + l * d.layer_stride + h, hv = d.v_head0 + l * d.layer_stride + h;
     groups[g] = WsGroup{s, l, h, g, 1, hk, hv, 0};
-    items[g] = WsItem{g, 0, cap_rows, 0};
+    items[g] = WsItem{g, 0, cap_rows, g};
     hg[((size_t)l * d.n_kv_heads + h) * d.n_seqs + s] = g;
     (void)heads;
   }
