@@ -66,7 +66,12 @@ struct Heads {
 constexpr int kHeadThreads = 256;
 constexpr int kVecPass = 32;  // query vectors (sequences x G) per pass
 constexpr int kWLd = 132;     // padded row stride (floats) of a staged basis: conflict-free row reads
-constexpr int kZLd = 36;      // row stride of the transposed rank-space averages
+// row stride of the transposed rank-space averages of a combine pass of VP vectors (odd:
+// the per-channel writes are conflict-free; the reads are broadcasts)
+template <int VP>
+__host__ __device__ constexpr int combine_zld() {
+  return VP + 1;
+}
 
 __host__ __device__ constexpr size_t qproj_smem_bytes() {
   return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd);
@@ -75,7 +80,7 @@ constexpr int kWtChunk = 64;  // chunk weights held in shared memory per vector 
 constexpr int kCombineVP = 16;  // query vectors per combine CTA (a head's sequences spread over CTAs)
 template <int VP>
 __host__ __device__ constexpr size_t combine_smem_bytes() {
-  return sizeof(float) * ((size_t)kD * kZLd + kD + (size_t)VP * kWtChunk);
+  return sizeof(float) * ((size_t)kD * combine_zld<VP>() + kD + (size_t)VP * kWtChunk);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -760,7 +765,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
 template <int G, int VP>
 __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   constexpr int SPP = VP / G > 0 ? VP / G : 1;
-  static_assert(VP % 8 == 0 && VP <= kZLd, "combine pass width");
+  static_assert(VP % 8 == 0, "combine pass width");
+  constexpr int kZLd = combine_zld<VP>();
   extern __shared__ __align__(16) float csm[];
   float* Zs = csm;                  // [kD][kZLd]   zbar of this pass, [channel][vector]
   float* mus = Zs + kD * kZLd;      // [kD]         mu_V

@@ -677,7 +677,7 @@ extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, 
 // (r_K, r_V), so that the warps working at the same time run the same code.
 // ----------------------------------------------------------------------------------------
 namespace {
-constexpr long long kItemMin = 16 * 1024, kItemMax = 256 * 1024;
+constexpr long long kItemMin = 16 * 1024, kItemMax = 128 * 1024;
 constexpr long long kScanWarps = 152 * 16;  // resident scan warps: 152 SMs x 4 CTAs x 4 warps
 constexpr long long kGuide = 2;
 constexpr long long kMaxChunks = 32;

@@ -10,7 +10,7 @@ import pytest
 
 from paper_2609_24298_gb300 import cobra
 
-ITEM_MIN, ITEM_MAX = 16 * 1024, 256 * 1024
+ITEM_MIN, ITEM_MAX = 16 * 1024, 128 * 1024
 
 
 @pytest.fixture(scope="module", autouse=True)
