@@ -390,29 +390,28 @@ def run_cobra(args):
                                  x_stride_head=128) for side in (0, 1)]
     block, cache = wl.dev.block, wl.dev.cache
 
-    stages = ("append_k", "append_v", "qproj", "scan", "combine")
+    stages = ("append_v", "qproj_append_k", "scan", "combine")
 
-    def step(ev=None):
-        # ev: 6 events bracketing the 5 launches (recorded on the launch stream)
-        if ev is not None:
-            ev[0].record(stream)
-        cobra.cobra_append(block, adesc[0], xk, pos, cache, None, stream)
-        if ev is not None:
-            ev[1].record(stream)
+    def step():
+        # one decode step through the public entry point: V append, query projection fused
+        # with the K append, scan, combine
+        cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], xk, xv, pos, q, cache, lens, None, out, ws,
+                                nbytes_ws, stream)
+
+    def staged_step(ev):
+        # the same launches as separate calls, with events between them (they serialise the
+        # launches, so this pass only gives the per-launch breakdown)
+        ev[0].record(stream)
         cobra.cobra_append(block, adesc[1], xv, pos, cache, None, stream)
-        if ev is not None:
-            ev[2].record(stream)
-        cobra.cobra_decode_qproj(block, desc, info, q, ws, nbytes_ws, stream)
-        if ev is not None:
-            ev[3].record(stream)
+        ev[1].record(stream)
+        cobra.cobra_decode_qproj_append(block, desc, info, q, adesc[0], xk, pos, cache, None, ws, nbytes_ws, stream)
+        ev[2].record(stream)
         cobra.cobra_decode_scan(block, desc, info, cache, lens, None, ws, nbytes_ws, stream)
-        if ev is not None:
-            ev[4].record(stream)
+        ev[3].record(stream)
         cobra.cobra_decode_combine(block, desc, info, lens, out, ws, nbytes_ws, stream)
-        if ev is not None:
-            ev[5].record(stream)
+        ev[4].record(stream)
 
-    launches_per_step = 5
+    launches_per_step = 4
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
@@ -443,7 +442,7 @@ def run_cobra(args):
     KB = min(K, 200)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(stages) + 1)] for _ in range(KB)]
     for k in range(KB):
-        step(ev[k])
+        staged_step(ev[k])
     torch.cuda.synchronize()
     stage_ms = {name: float(np.mean([e[i].elapsed_time(e[i + 1]) for e in ev])) for i, name in enumerate(stages)}
     scan_ms = stage_ms["scan"]
@@ -469,9 +468,8 @@ def run_cobra(args):
         xk.copy_(hk, non_blocking=True)
         xv.copy_(hv, non_blocking=True)
         q.copy_(hq, non_blocking=True)
-        cobra.cobra_append(block, adesc[0], xk, pos, cache, None, stream)
-        cobra.cobra_append(block, adesc[1], xv, pos, cache, None, stream)
-        cobra.cobra_decode_attn(block, desc, info, q, cache, lens, None, out, ws, nbytes_ws, stream)
+        cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], xk, xv, pos, q, cache, lens, None, out, ws,
+                                nbytes_ws, stream)
         hout.copy_(out, non_blocking=True)
 
     for _ in range(5):

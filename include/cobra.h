@@ -263,6 +263,26 @@ cobra_status cobra_decode_scan(const void* params, const cobra_decode_desc* desc
 cobra_status cobra_decode_combine(const void* params, const cobra_decode_desc* desc, const cobra_decode_info* info,
                                   const int* seq_lens, float* out, void* workspace, size_t ws_bytes, void* stream);
 
+/* The query projection fused with the K-side append of Table alg:kvrobin step 7 for one new
+ * token per sequence (both project through W_K): kdesc describes the K heads of `desc`
+ * (side 0, same head0 = desc->k_head0, layer_stride, n_layers, n_kv_heads and n_seqs, else
+ * COBRA_EINVAL); k_new, pos, cache and page_table as for cobra_append.  One launch. */
+cobra_status cobra_decode_qproj_append(const void* params, const cobra_decode_desc* desc, const cobra_decode_info* info,
+                                       const void* q, const cobra_compress_desc* kdesc, const void* k_new,
+                                       const int* pos, uint8_t* cache, const int* page_table, void* workspace,
+                                       size_t ws_bytes, void* stream);
+
+/* One decode step: append the new token's K and V codes of every (layer, kv-head, sequence)
+ * at pos[s] (Table alg:kvrobin step 7), then decode attention over seq_lens[s] tokens (which
+ * normally include the appended one).  kdesc / vdesc describe the K / V heads of `desc`
+ * (sides 0 / 1, head0 = desc->k_head0 / desc->v_head0, the other counts equal, else
+ * COBRA_EINVAL).  Four launches on `stream`: V append, query projection with the K append,
+ * scan, combine; nothing is synchronised. */
+cobra_status cobra_decode_step(const void* params, const cobra_decode_desc* desc, const cobra_decode_info* info,
+                               const cobra_compress_desc* kdesc, const cobra_compress_desc* vdesc, const void* k_new,
+                               const void* v_new, const int* pos, const void* q, uint8_t* cache, const int* seq_lens,
+                               const int* page_table, float* out, void* workspace, size_t ws_bytes, void* stream);
+
 /* ---------------------------------------------------------------------------------------
  * Decode attention without any device allocation.  (The paper has no counterpart; this is an
  * interface convenience.)

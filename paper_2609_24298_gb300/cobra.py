@@ -72,6 +72,13 @@ SIGNATURES = {
     "cobra_decode_workspace_size": (c_int, [ctypes.POINTER(DecodeDesc), P_int, P_int, P_int, P_size]),
     "cobra_decode_plan": (c_int, [ctypes.POINTER(DecodeDesc), P_int, P_int, P_int, c_void_p, c_size_t,
                                   ctypes.POINTER(DecodeInfo), c_void_p]),
+    "cobra_decode_qproj_append": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo), c_void_p,
+                                          ctypes.POINTER(CompressDesc), c_void_p, c_void_p, c_void_p, c_void_p,
+                                          c_void_p, c_size_t, c_void_p]),
+    "cobra_decode_step": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo),
+                                  ctypes.POINTER(CompressDesc), ctypes.POINTER(CompressDesc), c_void_p, c_void_p,
+                                  c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_size_t,
+                                  c_void_p]),
     "cobra_decode_plan_host": (c_int, [ctypes.POINTER(DecodeDesc), P_int, P_int, P_int, c_void_p, c_size_t, P_size,
                                        ctypes.POINTER(DecodeInfo)]),
     "cobra_decode_attn": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo), c_void_p,
@@ -307,6 +314,23 @@ def cobra_decode_plan_host(desc: DecodeDesc, head_r, head_b, seq_cap):
                                       ctypes.byref(info))
     _chk("cobra_decode_plan_host", st)
     return img, info
+
+
+def cobra_decode_qproj_append(params, desc: DecodeDesc, info: DecodeInfo, q, kdesc: CompressDesc, k_new, pos, cache,
+                              page_table, workspace, ws_bytes: int, stream=None):
+    st = lib().cobra_decode_qproj_append(_ptr(params), ctypes.byref(desc), ctypes.byref(info), _ptr(q),
+                                         ctypes.byref(kdesc), _ptr(k_new), _ptr(pos), _ptr(cache), _ptr(page_table),
+                                         _ptr(workspace), int(ws_bytes), _stream(stream))
+    _chk("cobra_decode_qproj_append", st)
+
+
+def cobra_decode_step(params, desc: DecodeDesc, info: DecodeInfo, kdesc: CompressDesc, vdesc: CompressDesc, k_new,
+                      v_new, pos, q, cache, seq_lens, page_table, out, workspace, ws_bytes: int, stream=None):
+    st = lib().cobra_decode_step(_ptr(params), ctypes.byref(desc), ctypes.byref(info), ctypes.byref(kdesc),
+                                 ctypes.byref(vdesc), _ptr(k_new), _ptr(v_new), _ptr(pos), _ptr(q), _ptr(cache),
+                                 _ptr(seq_lens), _ptr(page_table), _ptr(out), _ptr(workspace), int(ws_bytes),
+                                 _stream(stream))
+    _chk("cobra_decode_step", st)
 
 
 def cobra_decode_attn(params, desc: DecodeDesc, info: DecodeInfo, q, cache, seq_lens, page_table, out, workspace,

@@ -66,60 +66,50 @@ __device__ __forceinline__ void pack_piece(const uint8_t* codes, int ldc, int si
 
 // a8: single-token append.  One CTA of 8 warps per (layer, kv head): the head's basis is staged
 // in shared memory once (row stride kAppendWLd floats, so that a warp's 16-byte row reads are
-// conflict-free) and each warp appends the token of one sequence at a time.
+// conflict-free) and each warp appends the token of one sequence at a time.  The same steps run
+// inside the query projection for the K side (both project through W_K), see qproj_kernel.
 constexpr int kAppendThreads = 256;
 constexpr int kAppendWLd = 132;
 __host__ __device__ constexpr size_t append_smem_bytes() {
   return sizeof(float) * ((size_t)kD * kAppendWLd + (size_t)(kAppendThreads / 32) * kD + kD);
 }
 
-__global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) {
-  extern __shared__ __align__(16) float apsm[];
-  float* Ws = apsm;                     // [kD][kAppendWLd]
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  float* wmu = Ws + kD * kAppendWLd + (kAppendThreads / 32) * kD;  // W^T mu
-  float* xs = Ws + kD * kAppendWLd + warp * kD;
-  grid_dep_launch();
-  const int layer = blockIdx.x / a.n_kv, kv = blockIdx.x % a.n_kv;
-  const HeadEntry he = head_table(a.block)[a.head0 + layer * a.layer_stride + kv];
-  const int r = he.r, b = he.b;
-  if (r == 0) {
-    grid_dep_wait();
-    return;
-  }
-  const float* pool = param_pool(a.block);
-  // the basis and W^T mu (r floats; the pool is padded to 32 floats, so whole 16-byte chunks
-  // stay in it) are parameters: their copies start before the wait for the kernel ahead
-  if (threadIdx.x < (r + 3) / 4) cp_async16(smem_addr(wmu + 4 * threadIdx.x), pool + he.wmu_off + 4 * threadIdx.x);
-  stage_basis_issue(pool + he.w_off, r, kAppendWLd, Ws);
-  // the tokens, positions and the cache may be produced or read by the kernels ahead
-  grid_dep_wait();
-  // the first sequence's token and position are loaded while the basis arrives
-  __nv_bfloat16 xr[4];
-  int p_next = 0;
-  if (warp < a.n_seqs) {
-    const __nv_bfloat16* xp = a.x + layer * a.sl + warp * a.ss + kv * a.sh;
+// The new token and position of the warp's first sequence, loaded before the basis is waited for.
+struct AppendNext {
+  __nv_bfloat16 x[4];
+  int pos;
+};
+__device__ __forceinline__ AppendNext append_load(const CompressArgs& a, int layer, int kv, int seq) {
+  AppendNext n{};
+  if (seq < a.n_seqs) {
+    const __nv_bfloat16* xp = a.x + layer * a.sl + seq * a.ss + kv * a.sh;
+    const int lane = threadIdx.x & 31;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) xr[k] = xp[lane + 32 * k];
-    p_next = a.pos[warp];
+    for (int k = 0; k < 4; ++k) n.x[k] = xp[lane + 32 * k];
+    n.pos = a.pos[seq];
   }
-  cp_async_wait_all();
-  __syncthreads();
+  return n;
+}
+
+// Projects, quantises and writes the new token of sequences warp, warp + nwarps, ... of one head
+// (he, at (layer, kv)): y = W^T x - W^T mu from the staged basis Ws (row i = channel i, stride
+// kAppendWLd) and wmu, codes into the token's bits of its row with atomics (the row's other
+// tokens are untouched).  xs: 128 floats of the warp's shared memory; nx: the first sequence's
+// token, from append_load.
+__device__ __forceinline__ void append_tokens(const CompressArgs& a, const HeadEntry& he, int layer, int kv,
+                                              const float* Ws, const float* wmu, float* xs, int warp, int nwarps,
+                                              AppendNext nx) {
+  const int lane = threadIdx.x & 31;
+  const int r = he.r, b = he.b;
   const uint32_t rb = 16u * r * b;
   const float inv_delta = he.inv_delta, half = (float)(1 << (b - 1));
   const int cmax = (1 << b) - 1;
-  for (int seq = warp; seq < a.n_seqs; seq += kAppendThreads / 32) {
+  for (int seq = warp; seq < a.n_seqs; seq += nwarps) {
 #pragma unroll
-    for (int k = 0; k < 4; ++k) xs[lane + 32 * k] = __bfloat162float(xr[k]);
-    const int p = p_next;
+    for (int k = 0; k < 4; ++k) xs[lane + 32 * k] = __bfloat162float(nx.x[k]);
+    const int p = nx.pos;
     // the next sequence's token and position, in flight during this one's projection
-    const int nseq = seq + kAppendThreads / 32;
-    if (nseq < a.n_seqs) {
-      const __nv_bfloat16* xp = a.x + layer * a.sl + nseq * a.ss + kv * a.sh;
-#pragma unroll
-      for (int k = 0; k < 4; ++k) xr[k] = xp[lane + 32 * k];
-      p_next = a.pos[nseq];
-    }
+    nx = append_load(a, layer, kv, seq + nwarps);
     __syncwarp();
     const int row = p >> 7, tt = p & 127;
     const bool in_range = p >= 0 && (a.page_table ? (row >> 1) < a.pages_per_seq : row < a.rows_per_seq);
@@ -164,6 +154,33 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) 
     }
     __syncwarp();  // xs is rewritten for the next sequence
   }
+}
+
+__global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) {
+  extern __shared__ __align__(16) float apsm[];
+  float* Ws = apsm;                     // [kD][kAppendWLd]
+  const int warp = threadIdx.x >> 5;
+  float* wmu = Ws + kD * kAppendWLd + (kAppendThreads / 32) * kD;  // W^T mu
+  float* xs = Ws + kD * kAppendWLd + warp * kD;
+  grid_dep_launch();
+  const int layer = blockIdx.x / a.n_kv, kv = blockIdx.x % a.n_kv;
+  const HeadEntry he = head_table(a.block)[a.head0 + layer * a.layer_stride + kv];
+  if (he.r == 0) {
+    grid_dep_wait();
+    return;
+  }
+  const float* pool = param_pool(a.block);
+  // the basis and W^T mu (r floats; the pool is padded to 32 floats, so whole 16-byte chunks
+  // stay in it) are parameters: their copies start before the wait for the kernel ahead
+  if (threadIdx.x < (he.r + 3) / 4)
+    cp_async16(smem_addr(wmu + 4 * threadIdx.x), pool + he.wmu_off + 4 * threadIdx.x);
+  stage_basis_issue(pool + he.w_off, he.r, kAppendWLd, Ws);
+  // the tokens, positions and the cache may be produced or read by the kernels ahead
+  grid_dep_wait();
+  const AppendNext nx = append_load(a, layer, kv, warp);  // in flight while the basis arrives
+  cp_async_wait_all();
+  __syncthreads();
+  append_tokens(a, he, layer, kv, Ws, wmu, xs, warp, kAppendThreads / 32, nx);
 }
 
 }  // namespace cobra

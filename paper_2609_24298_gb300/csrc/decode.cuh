@@ -26,6 +26,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "compress.cuh"
 
 namespace cobra {
 
@@ -74,8 +75,9 @@ __host__ __device__ constexpr int combine_zld() {
 }
 
 __host__ __device__ constexpr size_t qproj_smem_bytes() {
-  return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd);
+  return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd + kD);
 }
+static_assert(kWLd == kAppendWLd, "the query projection stages W_K as the append reads it");
 constexpr int kWtChunk = 64;  // chunk weights held in shared memory per vector and round
 constexpr int kCombineVP = 16;  // query vectors per combine CTA (a head's sequences spread over CTAs)
 template <int VP>
@@ -88,15 +90,18 @@ __host__ __device__ constexpr size_t combine_smem_bytes() {
 //   q~_g = (Delta_K / sqrt d) log2(e) W_K^T q_g per query head, scaled by a power of two so
 //   that max |q~| of the group lands in [256, 512), split into fp16 hi + lo and laid out as
 //   the scan's MMA B fragments; Qsum_g = sum over channels of the fed hi + lo values.
+//   With ak.x set, the CTA first appends the new K token of every sequence of its head (a8),
+//   which projects through the same staged W_K.
 // ---------------------------------------------------------------------------------------
 template <int G>
-__global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
+__global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a, CompressArgs ak) {
   grid_dep_launch();
   constexpr int NTK = Heads<G>::NTK, SPP = kVecPass / G;
   extern __shared__ __align__(16) float qsm[];
   float* Ws = qsm;                  // [kD][kWLd]   W_K row i = channel i
-  float* Qs = Ws + kD * kWLd;       // [kVecPass][kD] queries of this pass (fp32)
+  float* Qs = Ws + kD * kWLd;       // [kVecPass][kD] queries of this pass (fp32); the appended tokens first
   float* Os = Qs + kVecPass * kD;   // [kVecPass][kWLd] scaled q~ of this pass
+  float* wmu = Os + kVecPass * kWLd;  // [kD] W_K^T mu_K for the append
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
   const int S = wh->n_seqs;
@@ -107,14 +112,22 @@ __global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a) {
   const int r = hk.r, layer = g0.layer, kv = g0.kv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const float scale = hk.delta * 0.088388347648318440f * 1.4426950408889634f;  // Delta/sqrt(128)*log2(e)
-  // the basis is a parameter: its copy overlaps the end of the kernel ahead; the queries and
-  // the q~ blocks of the workspace are touched only after the wait
+  // the basis is a parameter: its copy overlaps the end of the kernel ahead; the queries, the
+  // new tokens, the cache and the q~ blocks of the workspace are touched only after the wait
+  const bool append = ak.x != nullptr && r > 0;
+  if (append && tid < (r + 3) / 4) cp_async16(smem_addr(wmu + 4 * tid), pool + hk.wmu_off + 4 * tid);
   stage_basis_issue(pool + hk.w_off, r, kWLd, Ws);
   grid_dep_wait();
+  if (append) {
+    const AppendNext nx = append_load(ak, layer, kv, warp);
+    cp_async_wait_all();
+    __syncthreads();
+    append_tokens(ak, hk, layer, kv, Ws, wmu, Qs + warp * kD, warp, kHeadThreads / 32, nx);
+  }
   cp_async_wait_all();
   for (int s0 = 0; s0 < S; s0 += SPP) {
     const int ns = min(SPP, S - s0), nv = ns * G;
-    __syncthreads();  // basis staged; the previous pass is done with Qs and Os
+    __syncthreads();  // basis staged; the appends and the previous pass are done with Qs and Os
     // queries are only 2-byte aligned in general: element loads, all issued together
 #pragma unroll 16
     for (int idx = tid; idx < nv * kD; idx += kHeadThreads) {
@@ -763,7 +776,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
 // ---------------------------------------------------------------------------------------
 // One CTA per (layer, kv head) and run of VP / G sequences (VP query vectors).
 template <int G, int VP>
-__global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
+__global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) {
   constexpr int SPP = VP / G > 0 ? VP / G : 1;
   static_assert(VP % 8 == 0, "combine pass width");
   constexpr int kZLd = combine_zld<VP>();
@@ -772,7 +785,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   float* mus = Zs + kD * kZLd;      // [kD]         mu_V
   float* wts = mus + kD;            // [VP][kWtChunk] normalised chunk weights
   __shared__ float vinfo_m[VP], vinfo_inv_l[VP];
-  __shared__ int vinfo_first[VP], vinfo_n[VP], vinfo_g[VP];
+  __shared__ int vinfo_first[VP], vinfo_n[VP], vinfo_g[VP], vinfo_seq[VP];
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
   const float* parts = reinterpret_cast<const float*>(a.ws + wh->part_off);
@@ -791,18 +804,27 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
   // they are pulled into L2 here, while the scan ahead of this kernel is still finishing
   const float4* W4 = reinterpret_cast<const float4*>(pool + hv.w_off);
   for (int idx = tid; idx < rv * (kD / 32); idx += kHeadThreads) prefetch_l2(pool + hv.w_off + 32 * idx);
+  // the plan side of every vector: its group's chunks and query head
+  const int s0 = chunk * SPP;
+  const int ns = min(SPP, S - s0), nv = ns * G;
+  if (tid < nv) {
+    const WsGroup gr = groups[hg[s0 + tid / G]];
+    vinfo_first[tid] = gr.first_item;
+    vinfo_n[tid] = gr.n_items;
+    vinfo_g[tid] = tid % G;
+    vinfo_seq[tid] = gr.seq;
+  }
   // the appends of the next step may start their parameter staging meanwhile
   grid_dep_launch();
   // everything above is independent of the scan; its partials are read only from here on
   grid_dep_wait();
   {
-    const int s0 = chunk * SPP;
-    const int ns = min(SPP, S - s0), nv = ns * G;
-    __syncthreads();  // mu_V staged
-    // (1) per vector (warp w: vectors w, w + 8, w + 16, w + 24): m* = max over the chunks and
+    __syncthreads();  // mu_V and the vector table staged
+    // (1) per vector (warp w: vectors w, w + 8, ...): m* = max over the chunks and
     //     l* = sum 2^(m - m*) l, lanes over chunks, merged online (a chunk with no tokens has
-    //     m = -inf and no value entries; its weight is zero).  The four vectors' loads are
-    //     issued together.
+    //     m = -inf and no value entries; its weight is zero).  The vectors' loads are issued
+    //     together; the lanes keep the m of the first kWtChunk chunks and turn them into the
+    //     weights 2^(m - m*) / l* of the first round of (2).
     const int warp = tid >> 5, lane = tid & 31;
     constexpr int NU = VP / (kHeadThreads / 32);
     {
@@ -813,17 +835,11 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
 #pragma unroll
       for (int u = 0; u < NU; ++u) {
         const int v = warp + 8 * u;
-        const WsGroup gr = groups[hg[s0 + min(v, nv - 1) / G]];
-        ni[u] = (v < nv && a.seq_lens[gr.seq] > 0) ? gr.n_items : 0;
-        pg0[u] = parts + (size_t)gr.first_item * wh->part_stride + (v % G) * wh->g_stride;
+        ni[u] = (v < nv && a.seq_lens[vinfo_seq[v]] > 0) ? vinfo_n[v] : 0;
+        pg0[u] = parts + (v < nv ? (size_t)vinfo_first[v] * wh->part_stride + (v % G) * wh->g_stride : 0);
         M[u] = -INFINITY;
         Lsum[u] = 0.f;
         kmax = max(kmax, ni[u]);
-        if (v < nv && lane == 0) {
-          vinfo_first[v] = ni[u] > 0 ? gr.first_item : -1;
-          vinfo_n[v] = ni[u];
-          vinfo_g[v] = v % G;
-        }
       }
       for (int k = lane; k < kmax; k += 32) {
         float mk[NU], lk[NU];
@@ -835,6 +851,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
         }
 #pragma unroll
         for (int u = 0; u < NU; ++u) {
+          if (k < kWtChunk && warp + 8 * u < nv) wts[(warp + 8 * u) * kWtChunk + k] = mk[u];
           if (mk[u] == -INFINITY) continue;
           const float mn = fmaxf(M[u], mk[u]);
           Lsum[u] = Lsum[u] * exp2f(M[u] - mn) + lk[u] * exp2f(mk[u] - mn);
@@ -853,46 +870,61 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
           }
         }
         const int v = warp + 8 * u;
-        if (v < nv && lane == 0) {
+        if (v >= nv) continue;
+        const float inv_l = ni[u] > 0 ? 1.f / Lsum[u] : 0.f;
+        if (lane == 0) {
+          vinfo_first[v] = ni[u] > 0 ? vinfo_first[v] : -1;
+          vinfo_n[v] = ni[u];
           vinfo_m[v] = M[u];
-          vinfo_inv_l[v] = ni[u] > 0 ? 1.f / Lsum[u] : 0.f;
+          vinfo_inv_l[v] = inv_l;
+        }
+        // the same lane wrote wts[v][k] above for k < kmax
+        for (int k = lane; k < kWtChunk; k += 32) {
+          const float mk = k < ni[u] ? wts[v * kWtChunk + k] : -INFINITY;
+          wts[v * kWtChunk + k] = mk != -INFINITY ? exp2f(mk - M[u]) * inv_l : 0.f;
         }
       }
     }
     __syncthreads();
     // (2) zbar[v][i] = Delta (sum_k w_k acc_k[i] - 2^{b-1} + 1/2) with w_k = 2^(m_k - m*) / l*.
-    //     Rounds of kWtChunk chunks: the weights of a round are computed one (vector, chunk) per
-    //     thread into shared memory; then thread (channel i, vector parity) sums over them in
-    //     blocks of 4 vectors x 8 chunks whose 32 loads are all issued before any is used.
+    //     Rounds of kWtChunk chunks (the first round's weights come from (1); later rounds
+    //     compute them one (vector, chunk) per thread into shared memory).  Thread (channel i,
+    //     group grp) of rw = r_V rounded up to 32, 64 or 128 channels owns the vectors
+    //     grp, grp + ng, ... (ng = 256 / rw groups) and sums over the chunks in blocks of
+    //     4 vectors x 8 chunks whose 32 loads are all issued before any is used.
     {
-      const int i = tid & (kD - 1), par = tid >> 7;
+      const int rw = rv <= 32 ? 32 : rv <= 64 ? 64 : kD;
+      const int ng = kHeadThreads / rw;
+      const int i = tid % rw, grp = tid / rw;
       int kmax = 0;
       for (int v = 0; v < nv; ++v) kmax = max(kmax, vinfo_n[v]);
       float acc[VP / 2];
 #pragma unroll
       for (int q = 0; q < VP / 2; ++q) acc[q] = 0.f;
       for (int k0 = 0; k0 < kmax; k0 += kWtChunk) {
-        __syncthreads();  // the previous round's weights are consumed
-        for (int idx = tid; idx < nv * kWtChunk; idx += kHeadThreads) {
-          const int v = idx / kWtChunk, k = k0 + idx % kWtChunk;
-          float w = 0.f;
-          if (k < vinfo_n[v]) {
-            const float mk = parts[(size_t)(vinfo_first[v] + k) * wh->part_stride + vinfo_g[v] * wh->g_stride];
-            if (mk != -INFINITY) w = exp2f(mk - vinfo_m[v]) * vinfo_inv_l[v];
+        if (k0 > 0) {
+          __syncthreads();  // the previous round's weights are consumed
+          for (int idx = tid; idx < nv * kWtChunk; idx += kHeadThreads) {
+            const int v = idx / kWtChunk, k = k0 + idx % kWtChunk;
+            float w = 0.f;
+            if (k < vinfo_n[v]) {
+              const float mk = parts[(size_t)(vinfo_first[v] + k) * wh->part_stride + vinfo_g[v] * wh->g_stride];
+              if (mk != -INFINITY) w = exp2f(mk - vinfo_m[v]) * vinfo_inv_l[v];
+            }
+            wts[idx] = w;
           }
-          wts[idx] = w;
+          __syncthreads();
         }
-        __syncthreads();
         if (i >= rv) continue;
         const int kr = min(kWtChunk, kmax - k0);
 #pragma unroll
         for (int q0 = 0; q0 < VP / 2; q0 += 4) {
-          if (2 * q0 + par >= nv) break;
+          if (grp + ng * q0 >= nv) break;
           for (int kb = 0; kb < kr; kb += 8) {
             float x[4][8];
 #pragma unroll
             for (int qq = 0; qq < 4; ++qq) {
-              const int v = 2 * (q0 + qq) + par;
+              const int v = grp + ng * (q0 + qq);
               const int n = v < nv ? vinfo_n[v] - k0 : 0;
               const float* px = parts + (size_t)max(vinfo_first[v < nv ? v : 0], 0) * wh->part_stride +
                                 (size_t)k0 * wh->part_stride + (v < nv ? vinfo_g[v] : 0) * wh->g_stride + 4 + i;
@@ -901,7 +933,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
             }
 #pragma unroll
             for (int qq = 0; qq < 4; ++qq) {
-              const int v = 2 * (q0 + qq) + par;
+              const int v = grp + ng * (q0 + qq);
               if (v >= nv) break;
               const float* wv = wts + v * kWtChunk + kb;
 #pragma unroll
@@ -913,11 +945,13 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
           }
         }
       }
+      if (i < rv) {
 #pragma unroll
-      for (int q = 0; q < VP / 2; ++q) {
-        const int v = 2 * q + par;
-        if (v >= nv) break;
-        Zs[i * kZLd + v] = (i < rv && vinfo_first[v] >= 0) ? hv.delta * (acc[q] - cen) : 0.f;
+        for (int q = 0; q < VP / 2; ++q) {
+          const int v = grp + ng * q;
+          if (v >= nv) break;
+          Zs[i * kZLd + v] = vinfo_first[v] >= 0 ? hv.delta * (acc[q] - cen) : 0.f;
+        }
       }
     }
     __syncthreads();
@@ -956,7 +990,7 @@ __global__ void __launch_bounds__(kHeadThreads) combine_kernel(DecodeArgs a) {
         const int vv = v0 + v;
         if (vv >= nv) break;
         const int seq = s0 + vv / G, g = vv % G;
-        const bool empty = a.seq_lens[groups[hg[seq]].seq] <= 0;
+        const bool empty = vinfo_first[vv] < 0;  // a sequence without tokens
         float* out = a.out + layer * a.o_sl + seq * a.o_ss + (long long)(kv * G + g) * kD + d0;
         const float4 y = empty ? make_float4(0.f, 0.f, 0.f, 0.f) : o[v];
         out[0] = y.x;  // the output is only 4-byte aligned in general

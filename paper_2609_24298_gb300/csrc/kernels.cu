@@ -189,14 +189,17 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), unsigned grid, unsigned block, 
 }
 }  // namespace
 
-extern "C" cobra_status cobra_append(const void* params, const cobra_compress_desc* d, const void* x, const int* pos,
-                                     uint8_t* cache, const int* page_table, void* stream) {
+namespace {
+// validated append arguments for one side
+cobra_status append_args(const void* params, const cobra_compress_desc* d, const void* x, const int* pos,
+                         uint8_t* cache, const int* page_table, CompressArgs& a) {
   cobra_status st = check_compress_desc(d);
   if (st != COBRA_OK) return st;
   if (!params || !x || !pos || !cache) return COBRA_EINVAL;
   if (!aligned(params, 256) || !aligned(cache, 256) || !aligned(x, 2)) return COBRA_EALIGN;
   if (page_table && d->pages_per_seq < 1) return COBRA_EINVAL;
-  CompressArgs a{};
+  if ((long long)d->n_layers * d->n_kv_heads > 0x7fffffffLL) return COBRA_EINVAL;
+  a = CompressArgs{};
   a.block = static_cast<const unsigned char*>(params);
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.cache = cache;
@@ -213,8 +216,16 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
   a.n_seqs = d->n_seqs;
   a.rows_per_seq = d->rows_per_seq;
   a.pages_per_seq = d->pages_per_seq;
+  return COBRA_OK;
+}
+}  // namespace
+
+extern "C" cobra_status cobra_append(const void* params, const cobra_compress_desc* d, const void* x, const int* pos,
+                                     uint8_t* cache, const int* page_table, void* stream) {
+  CompressArgs a;
+  cobra_status st = append_args(params, d, x, pos, cache, page_table, a);
+  if (st != COBRA_OK) return st;
   const long long grid = (long long)d->n_layers * d->n_kv_heads;  // one CTA per (layer, kv head)
-  if (grid > 0x7fffffffLL) return COBRA_EINVAL;
   static bool attr = false;
   if (!attr) {
     if (cudaFuncSetAttribute(append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_smem_bytes()) !=
@@ -234,7 +245,7 @@ enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
 template <int G>
 cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_items, int stages, cudaStream_t s,
-                           bool after_plan_kernel = false) {
+                           bool after_plan_kernel = false, const CompressArgs& ak = CompressArgs{}) {
   static bool head_attr = false;
   if (!head_attr) {
     if (cudaFuncSetAttribute(qproj_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)qproj_smem_bytes()) !=
@@ -248,9 +259,10 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
     // the query projection reads the plan before its wait; right after the plan kernel it is
     // launched in plain stream order
     if (after_plan_kernel) {
-      qproj_kernel<G><<<n_heads, kHeadThreads, qproj_smem_bytes(), s>>>(a);
+      qproj_kernel<G><<<n_heads, kHeadThreads, qproj_smem_bytes(), s>>>(a, ak);
       if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
-    } else if (launch_pdl(qproj_kernel<G>, (unsigned)n_heads, kHeadThreads, qproj_smem_bytes(), s, a) != cudaSuccess) {
+    } else if (launch_pdl(qproj_kernel<G>, (unsigned)n_heads, kHeadThreads, qproj_smem_bytes(), s, a, ak) !=
+               cudaSuccess) {
       return COBRA_ECUDA;
     }
   }
@@ -287,7 +299,8 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
 
 cobra_status decode_common(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info, const void* q,
                            const uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
-                           void* workspace, size_t ws_bytes, void* stream, int stages) {
+                           void* workspace, size_t ws_bytes, void* stream, int stages,
+                           const CompressArgs& ak = CompressArgs{}) {
   if (!d || !info || !params || !workspace) return COBRA_EINVAL;
   if ((stages & kQproj) && !q) return COBRA_EINVAL;
   if ((stages & kScan) && (!cache || !seq_lens)) return COBRA_EINVAL;
@@ -321,8 +334,20 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   cudaStream_t s = (cudaStream_t)stream;
   const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
   if (n_heads * d->n_seqs != info->n_groups) return COBRA_EINVAL;  // plan made for another descriptor
-  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s);
-  return launch_decode<8>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s);
+  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak);
+  return launch_decode<8>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak);
+}
+
+// K-side append arguments that match the decode descriptor's K heads
+cobra_status k_append_args(const void* params, const cobra_decode_desc* d, const cobra_compress_desc* kdesc,
+                           const void* k_new, const int* pos, uint8_t* cache, const int* page_table, CompressArgs& ak) {
+  if (!d || !kdesc) return COBRA_EINVAL;
+  cobra_status st = append_args(params, kdesc, k_new, pos, cache, page_table, ak);
+  if (st != COBRA_OK) return st;
+  if (kdesc->side != 0 || kdesc->head0 != d->k_head0 || kdesc->layer_stride != d->layer_stride ||
+      kdesc->n_layers != d->n_layers || kdesc->n_kv_heads != d->n_kv_heads || kdesc->n_seqs != d->n_seqs)
+    return COBRA_EINVAL;
+  return COBRA_OK;
 }
 }  // namespace
 
@@ -338,6 +363,38 @@ extern "C" cobra_status cobra_decode_attn(const void* params, const cobra_decode
 extern "C" cobra_status cobra_decode_qproj(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info,
                                            const void* q, void* workspace, size_t ws_bytes, void* stream) {
   return decode_common(params, d, info, q, nullptr, nullptr, nullptr, nullptr, workspace, ws_bytes, stream, kQproj);
+}
+
+extern "C" cobra_status cobra_decode_qproj_append(const void* params, const cobra_decode_desc* d,
+                                                  const cobra_decode_info* info, const void* q,
+                                                  const cobra_compress_desc* kdesc, const void* k_new, const int* pos,
+                                                  uint8_t* cache, const int* page_table, void* workspace,
+                                                  size_t ws_bytes, void* stream) {
+  CompressArgs ak;
+  cobra_status st = k_append_args(params, d, kdesc, k_new, pos, cache, page_table, ak);
+  if (st != COBRA_OK) return st;
+  st = decode_common(params, d, info, q, nullptr, nullptr, nullptr, nullptr, workspace, ws_bytes, stream, kQproj, ak);
+  return st != COBRA_OK ? st : launch_status();
+}
+
+extern "C" cobra_status cobra_decode_step(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info,
+                                          const cobra_compress_desc* kdesc, const cobra_compress_desc* vdesc,
+                                          const void* k_new, const void* v_new, const int* pos, const void* q,
+                                          uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
+                                          void* workspace, size_t ws_bytes, void* stream) {
+  if (!d || !vdesc || !q || !seq_lens || !out) return COBRA_EINVAL;
+  CompressArgs ak, av;
+  cobra_status st = k_append_args(params, d, kdesc, k_new, pos, cache, page_table, ak);
+  if (st != COBRA_OK) return st;
+  st = append_args(params, vdesc, v_new, pos, cache, page_table, av);
+  if (st != COBRA_OK) return st;
+  if (vdesc->side != 1 || vdesc->head0 != d->v_head0 || vdesc->layer_stride != d->layer_stride ||
+      vdesc->n_layers != d->n_layers || vdesc->n_kv_heads != d->n_kv_heads || vdesc->n_seqs != d->n_seqs)
+    return COBRA_EINVAL;
+  st = cobra_append(params, vdesc, v_new, pos, cache, page_table, stream);
+  if (st != COBRA_OK) return st;
+  return decode_common(params, d, info, q, cache, seq_lens, page_table, out, workspace, ws_bytes, stream,
+                       kQproj | kScan | kCombine, ak);
 }
 
 extern "C" cobra_status cobra_decode_scan(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info,

@@ -9,7 +9,8 @@ attend over identical codes: a legitimate boundary flip on a heavily weighted to
 the output by far more than the decode tolerance), and decode runs in the launch
 configuration the benchmark times (query projection, scan, combine on one stream) over the
 whole cache; sampled outputs must be within max relative error 2e-3 of the oracle's attention.
-The single-call entry point must reproduce the staged calls bit for bit."""
+The single-call entry points (decode attention; the decode step with both appends) must
+reproduce the staged calls bit for bit."""
 import numpy as np
 import pytest
 import torch
@@ -105,10 +106,24 @@ def run_workload(cfg, layers, params, srcs, lens, samples, paged=False, seed=5):
              for side in (0, 1)]
     block, cache, pt = wl.dev.block, wl.dev.cache, wl.page_table
     stream = torch.cuda.current_stream()
+    before = cache.clone()
     cobra.cobra_append(block, adesc[0], xk, pos, cache, pt, stream)
     cobra.cobra_append(block, adesc[1], xv, pos, cache, pt, stream)
     torch.cuda.synchronize()
     assert cobra.cobra_check(stream) == cobra.COBRA_OK
+
+    # the one-call decode step (V append, query projection fused with the K append, scan,
+    # combine) writes the same cache bytes and the same outputs as the separate calls
+    step_out = torch.full((L, S, H * G, D), float("nan"), dtype=torch.float32, device=DEV)
+    cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], xk, xv, pos, q, before, lens_d, pt, step_out, ws,
+                            nws, stream)
+    staged_out = torch.full_like(step_out, float("nan"))
+    cobra.cobra_decode_attn(block, desc, info, q, cache, lens_d, pt, staged_out, ws, nws, stream)
+    torch.cuda.synchronize()
+    assert cobra.cobra_check(stream) == cobra.COBRA_OK
+    assert torch.equal(before, cache)
+    assert torch.equal(step_out, staged_out)
+    del before, step_out, staged_out
 
     # compress + append parity on the sampled heads, then the oracle's rows in their place
     hk, hv = xk.float().cpu().numpy(), xv.float().cpu().numpy()

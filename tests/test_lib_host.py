@@ -165,6 +165,21 @@ def test_argument_checks_reject_bad_input(L):
                            rows_per_seq=1)
     with pytest.raises(cobra.CobraError):
         cobra.cobra_decode_workspace_size(dd, np.array([2, 2]), np.array([1, 1]), np.array([10]))
+    # the decode step's append descriptors must describe the decode descriptor's K and V heads
+    d4 = cobra.decode_desc(k_head0=0, v_head0=1, layer_stride=1, n_layers=1, n_kv_heads=1, group=4, n_seqs=1,
+                           rows_per_seq=1)
+    info = cobra.DecodeInfo(1, 1, 16, 0)
+    kd = cobra.compress_desc(head0=0, layer_stride=1, n_layers=1, n_kv_heads=1, side=0, n_seqs=1, rows_per_seq=1)
+    vd = cobra.compress_desc(head0=1, layer_stride=1, n_layers=1, n_kv_heads=1, side=1, n_seqs=1, rows_per_seq=1)
+    kd_other = cobra.compress_desc(head0=1, layer_stride=1, n_layers=1, n_kv_heads=1, side=0, n_seqs=1,
+                                   rows_per_seq=1)
+    for k_, v_ in ((vd, vd), (kd, kd), (kd_other, vd)):
+        with pytest.raises(cobra.CobraError) as e:
+            cobra.cobra_decode_step(256, d4, info, k_, v_, 256, 256, 256, 256, 256, 256, None, 256, 256, 1 << 20)
+        assert e.value.status == cobra.COBRA_EINVAL
+    with pytest.raises(cobra.CobraError) as e:
+        cobra.cobra_decode_qproj_append(256, d4, info, 256, vd, 256, 256, 256, None, 256, 1 << 20)
+    assert e.value.status == cobra.COBRA_EINVAL
 
 
 def test_decode_plan_sizes(L):
