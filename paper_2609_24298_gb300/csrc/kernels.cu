@@ -13,6 +13,7 @@
 #include "compress.cuh"
 #include "compress_tc.cuh"
 #include "decode.cuh"
+#include "decode_heads.cuh"
 
 using namespace cobra;
 
