@@ -379,9 +379,15 @@ def run_cobra(args):
     # per-step inputs: the new token's K and V for every (layer, kv head, seq); the queries
     gen = torch.Generator(device=dev)
     gen.manual_seed(2609 + rank)
-    xk = torch.randn((L, S, H, 128), generator=gen, device=dev).to(torch.bfloat16)
-    xv = torch.randn((L, S, H, 128), generator=gen, device=dev).to(torch.bfloat16)
-    q = torch.randn((L, S, Hq, 128), generator=gen, device=dev).to(torch.bfloat16)
+    # the step's inputs (new K and V tokens, queries) in one device buffer, so that the
+    # end-to-end leg moves them with one host-to-device copy
+    n_kv, n_q = L * S * H * 128, L * S * Hq * 128
+    din = torch.empty(2 * n_kv + n_q, dtype=torch.bfloat16, device=dev)
+    xk, xv, q = (din[:n_kv].view(L, S, H, 128), din[n_kv:2 * n_kv].view(L, S, H, 128),
+                 din[2 * n_kv:].view(L, S, Hq, 128))
+    xk.copy_(torch.randn((L, S, H, 128), generator=gen, device=dev))
+    xv.copy_(torch.randn((L, S, H, 128), generator=gen, device=dev))
+    q.copy_(torch.randn((L, S, Hq, 128), generator=gen, device=dev))
     out = torch.empty((L, S, Hq, 128), dtype=torch.float32, device=dev)
     pos = torch.full((S,), T - 1, dtype=torch.int32, device=dev)
     lens = torch.full((S,), T, dtype=torch.int32, device=dev)
@@ -455,19 +461,13 @@ def run_cobra(args):
     value = weak_scaling_gbs(bytes_step, K, world, total_ms)
 
     # end to end through the public API: pinned host inputs in, host output out, every step
-    hk = torch.empty_like(xk, device="cpu").pin_memory()
-    hv = torch.empty_like(xv, device="cpu").pin_memory()
-    hq = torch.empty_like(q, device="cpu").pin_memory()
+    hin = torch.empty_like(din, device="cpu").pin_memory()
     hout = torch.empty_like(out, device="cpu").pin_memory()
-    hk.copy_(xk.cpu())
-    hv.copy_(xv.cpu())
-    hq.copy_(q.cpu())
+    hin.copy_(din.cpu())
     Ke = max(10, K // 4)
 
     def e2e_step():
-        xk.copy_(hk, non_blocking=True)
-        xv.copy_(hv, non_blocking=True)
-        q.copy_(hq, non_blocking=True)
+        din.copy_(hin, non_blocking=True)
         cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], xk, xv, pos, q, cache, lens, None, out, ws,
                                 nbytes_ws, stream)
         hout.copy_(out, non_blocking=True)
@@ -483,14 +483,14 @@ def run_cobra(args):
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / Ke
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
-    h2d = (xk.numel() + xv.numel() + q.numel()) * 2
+    h2d = din.numel() * 2
     d2h = out.numel() * 4
 
     peak, peak_kind = hbm_peak()
     achieved = bytes_step / (scan_ms * 1e-3) / 1e9
     compress = None
     if not args.no_compress:
-        del hk, hv, hq, hout
+        del hin, hout
         compress = run_compress_leg(args, dev, stream, peak)
     traffic = profiled_traffic()
     if rank == 0:
