@@ -103,6 +103,22 @@ __device__ __forceinline__ void bulk_g2s_if(bool p, uint32_t dst, const void* sr
       "l"(src), "r"(bytes), "r"(bar), "r"((int)p)
       : "memory");
 }
+// One lane's refill of a ring stage with a K row and a V row on one mbarrier, under one
+// predicate: the proxy fence (the warp's generic reads of the stage are ordered before the
+// async copies that overwrite it), arrive.expect_tx of both sizes, then the two bulk copies
+// (a size of 0 skips that copy).
+__device__ __forceinline__ void refill_pair_if(bool p, uint32_t bar, uint32_t dst_k, const void* src_k, uint32_t kb,
+                                               uint32_t dst_v, const void* src_v, uint32_t vb) {
+  asm volatile(
+      "{\n .reg .pred q, qk, qv;\n setp.ne.b32 q, %8, 0;\n"
+      " setp.ne.and.b32 qk, %3, 0, q;\n setp.ne.and.b32 qv, %6, 0, q;\n"
+      " @q fence.proxy.async.shared::cta;\n"
+      " @q mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %7;\n"
+      " @qk cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%1], [%2], %3, [%0];\n"
+      " @qv cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%4], [%5], %6, [%0];\n}\n" ::"r"(bar),
+      "r"(dst_k), "l"(src_k), "r"(kb), "r"(dst_v), "l"(src_v), "r"(vb), "r"(kb + vb), "r"((int)p)
+      : "memory");
+}
 __device__ __forceinline__ void fence_proxy_async_smem_if(bool p) {
   asm volatile("{\n .reg .pred q;\n setp.ne.b32 q, %0, 0;\n @q fence.proxy.async.shared::cta;\n}\n" ::"r"((int)p)
                : "memory");

@@ -368,24 +368,32 @@ __device__ __forceinline__ void scan_item(const DecodeArgs& a, ScanWarp& w, int 
   const float qscale = qhdr[8];
   const uint32_t one = a.one;
 
-  // issue state: next row and stage to load (every lane tracks it; lane 0 issues)
+  // issue state: next row and stage to load (every lane tracks it; lane 0 issues).  In a
+  // contiguous cache the item's rows follow one another, so the sources advance by a row;
+  // a paged cache looks each row's page up.
   int iss_row = row0, iss_stage = 0;
   const uint8_t* kbase = a.cache + koff;
   const uint8_t* vbase = a.cache + voff;
+  const int* const page_table = a.page_table;
+  const int pages_per_seq = a.pages_per_seq, seq = gr.seq;
+  const size_t slot0 = (size_t)seq * a.rows_per_seq + row0;
+  const uint8_t* ksrc = kbase + slot0 * rbk;
+  const uint8_t* vsrc = vbase + slot0 * rbv;
+  const uint32_t ring0 = smem_addr(w.ring), bar0 = smem_addr(w.bars);
+  const int nstage = w.nstage;
   auto issue_next = [&]() {
-    const uint32_t bar = smem_addr(&w.bars[iss_stage]);
-    const uint32_t dst = smem_addr(w.ring + (size_t)iss_stage * stage_bytes);
-    mbar_arrive_expect_tx_if(leader, bar, rbk + rbv);
-    if (rbk)
-      bulk_g2s_if(leader, dst,
-                  kbase + row_offset(0, rbk, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbk,
-                  bar);
-    if (rbv)
-      bulk_g2s_if(leader, dst + kst,
-                  vbase + row_offset(0, rbv, gr.seq, iss_row, a.page_table, a.pages_per_seq, a.rows_per_seq), rbv,
-                  bar);
+    const uint8_t* ks = ksrc;
+    const uint8_t* vs = vsrc;
+    if (page_table) {
+      ks = kbase + row_offset(0, rbk, seq, iss_row, page_table, pages_per_seq, 0);
+      vs = vbase + row_offset(0, rbv, seq, iss_row, page_table, pages_per_seq, 0);
+    }
+    const uint32_t dst = ring0 + (uint32_t)(iss_stage * stage_bytes);
+    refill_pair_if(leader, bar0 + 8u * iss_stage, dst, ks, rbk, dst + kst, vs, rbv);
+    ksrc += rbk;
+    vsrc += rbv;
     ++iss_row;
-    if (++iss_stage == w.nstage) iss_stage = 0;
+    iss_stage = iss_stage + 1 == nstage ? 0 : iss_stage + 1;
   };
   int issued = min(n_loads, w.nstage);
   if (issued > 0 && rbk) {
@@ -414,8 +422,7 @@ __device__ __forceinline__ void scan_item(const DecodeArgs& a, ScanWarp& w, int 
     --w.outstanding;
     if (++w.wait_stage == w.nstage) w.wait_stage = 0;
     if (issued < n_loads) {
-      fence_proxy_async_smem_if(leader);
-      issue_next();
+      issue_next();  // its proxy fence orders this warp's reads of the stage before the copies
       ++issued;
       ++w.outstanding;
     }
