@@ -410,9 +410,11 @@ __device__ __forceinline__ void scan_item(const DecodeArgs& a, ScanWarp& w, int 
 
   // wait for the next stage; returns its buffer or nullptr on timeout
   auto acquire = [&]() -> const uint8_t* {
-    const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(smem_addr(&w.bars[w.wait_stage]),
-                                                              (w.phase_bits >> w.wait_stage) & 1u, kWaitLimitNs));
-    if (!ok) return nullptr;
+    const uint32_t bar = bar0 + 8u * w.wait_stage, parity = (w.phase_bits >> w.wait_stage) & 1u;
+    // the stage has normally landed already: one probe, and the bounded wait only when not
+    if (!__all_sync(0xffffffffu, mbar_try_wait(bar, parity)) &&
+        !__all_sync(0xffffffffu, mbar_wait_bounded(bar, parity, kWaitLimitNs)))
+      return nullptr;
     w.phase_bits ^= 1u << w.wait_stage;
     return w.ring + (size_t)w.wait_stage * stage_bytes;
   };
