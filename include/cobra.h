@@ -98,6 +98,19 @@ void cobra_alloc_opts_default(cobra_alloc_opts* o);
 cobra_status cobra_allocate(int n_heads, int d, const double* w, double bpd, const cobra_alloc_opts* opts,
                             int* r, int* b, double* budget, double* dist, long long* rate_bits);
 
+/* App. E "Exact DP over measured distortion": the exact DP of COBRA_ALLOC_EXACT run on
+ * explicit per-head distortion tables (e.g. from cobra_measure_distortion) instead of the
+ * surrogate.  D: host [n_heads][n_r][n_b] fp64, D[h][i][j] = head h's distortion at
+ * (r_list[i], b_list[j]); a row with r_list[i] = 0 means no codes (only its first entry is
+ * read).  r_list strictly ascending in [0, d], b_list strictly ascending in [1, 16].
+ * Minimises sum_h D_h subject to sum_h r_h b_h <= n_heads * d * bpd; per head and rate the
+ * smallest D is kept (the first in (r, b) order on ties), the final pick is the smallest
+ * total, then the fewest bits.  Outputs as cobra_allocate (dist may be NULL).  Errors:
+ * EINVAL (bad sizes, unsorted lists, non-finite D), EBUDGET (no feasible choice). */
+cobra_status cobra_allocate_tables(int n_heads, int d, int n_r, const int* r_list, int n_b, const int* b_list,
+                                   const double* D, double bpd, int* r_out, int* b_out, double* dist,
+                                   long long* rate_bits);
+
 /* ---------------------------------------------------------------------------------------
  * Calibration helpers (host, fp64).  Table alg:kvrobin steps 1, 2, 5, 6.
  * ------------------------------------------------------------------------------------- */

@@ -57,6 +57,8 @@ SIGNATURES = {
     "cobra_alloc_opts_default": (None, [ctypes.POINTER(AllocOpts)]),
     "cobra_allocate": (c_int, [c_int, c_int, P_double, c_double, ctypes.POINTER(AllocOpts), P_int, P_int, P_double,
                                P_double, P_ll]),
+    "cobra_allocate_tables": (c_int, [c_int, c_int, c_int, P_int, c_int, P_int, P_double, c_double, P_int, P_int,
+                                      P_double, P_ll]),
     "cobra_loading_factor": (c_int, [c_int, P_double]),
     "cobra_hadamard": (c_int, [c_int, P_i8, P_double]),
     "cobra_calibrate_head": (c_int, [c_int, c_int, P_float, c_int, P_float, P_double, P_double, P_double, P_double]),
@@ -174,6 +176,24 @@ def cobra_allocate(w, bpd: float, opts: AllocOpts | None = None):
                               dist.ctypes.data_as(P_double), ctypes.byref(rate))
     _chk("cobra_allocate", st)
     return dict(r=r, b=b, budget=bud, dist=dist, rate_bits=rate.value)
+
+
+def cobra_allocate_tables(tables, r_list, b_list, bpd: float, d: int = 128):
+    """Exact DP on explicit tables [n_heads][len(r_list)][len(b_list)] (App. E)."""
+    D, Dp = _np(np.ascontiguousarray(tables, dtype=np.float64), np.float64, c_double)
+    rl, rlp = _np(r_list, np.int32, c_int)
+    bl, blp = _np(b_list, np.int32, c_int)
+    n = D.shape[0]
+    if D.shape != (n, len(rl), len(bl)):
+        raise ValueError("tables must be [n_heads][len(r_list)][len(b_list)]")
+    r = np.zeros(n, np.int32)
+    b = np.zeros(n, np.int32)
+    dist = np.zeros(n, np.float64)
+    rate = c_ll(0)
+    st = lib().cobra_allocate_tables(n, int(d), len(rl), rlp, len(bl), blp, Dp, float(bpd), r.ctypes.data_as(P_int),
+                                     b.ctypes.data_as(P_int), dist.ctypes.data_as(P_double), ctypes.byref(rate))
+    _chk("cobra_allocate_tables", st)
+    return dict(r=r, b=b, dist=dist, rate_bits=rate.value)
 
 
 def cobra_loading_factor(b: int) -> float:

@@ -167,42 +167,38 @@ long long complete_alloc(const std::vector<Head>& H, std::vector<int>& r, std::v
   return slack;
 }
 
-// Exact DP over integer rates (App. E separable knapsack).
-cobra_status exact_dp(const std::vector<Head>& H, double B_tot, const Opts& o, const std::vector<int>& grid,
-                      std::vector<int>& r, std::vector<int>& b, std::vector<double>& D) {
-  const int n = (int)H.size();
+// Exact DP over integer rates (App. E separable knapsack), on per-head options.
+struct RateOpt {
+  long long rate;
+  double D;
+  int r, b;
+};
+
+// One option per distinct rate: the smallest D, the first in the given order on ties; sorted
+// by rate.
+std::vector<RateOpt> unique_by_rate(const std::vector<RateOpt>& all) {
+  std::vector<RateOpt> uniq;
+  for (const RateOpt& x : all) {
+    bool found = false;
+    for (RateOpt& u : uniq)
+      if (u.rate == x.rate) {
+        found = true;
+        if (x.D < u.D) u = x;
+        break;
+      }
+    if (!found) uniq.push_back(x);
+  }
+  std::stable_sort(uniq.begin(), uniq.end(), [](const RateOpt& a, const RateOpt& c) { return a.rate < c.rate; });
+  return uniq;
+}
+
+cobra_status dp_over_options(const std::vector<std::vector<RateOpt>>& opts, double B_tot, std::vector<int>& r,
+                             std::vector<int>& b, std::vector<double>& D) {
+  const int n = (int)opts.size();
   const long long cap = (long long)std::floor(B_tot + 1e-9);
   if (cap < 0 || cap > (1LL << 26)) return COBRA_EINVAL;
-  struct Opt {
-    long long rate;
-    double D;
-    int r, b;
-  };
-  std::vector<std::vector<Opt>> opts(n);
-  for (int h = 0; h < n; ++h) {
-    // one option per distinct rate: smallest D, first in (r asc, b asc) order on ties
-    std::vector<Opt> all;
-    for (int rr : grid) {
-      if (rr == 0) {
-        all.push_back({0, distortion(H[h], 0, 0), 0, 0});
-        continue;
-      }
-      for (int bb = o.b_min; bb <= o.b_max; ++bb) all.push_back({(long long)rr * bb, distortion(H[h], rr, bb), rr, bb});
-    }
-    std::vector<Opt> uniq;
-    for (const Opt& x : all) {
-      bool found = false;
-      for (Opt& u : uniq)
-        if (u.rate == x.rate) {
-          found = true;
-          if (x.D < u.D) u = x;
-          break;
-        }
-      if (!found) uniq.push_back(x);
-    }
-    std::stable_sort(uniq.begin(), uniq.end(), [](const Opt& a, const Opt& c) { return a.rate < c.rate; });
-    opts[h] = uniq;
-  }
+  for (const auto& o : opts)
+    if (o.size() > 32767) return COBRA_EINVAL;
   const double INF = std::numeric_limits<double>::infinity();
   std::vector<double> dp(cap + 1, INF), nw(cap + 1);
   dp[0] = 0.0;
@@ -211,7 +207,7 @@ cobra_status exact_dp(const std::vector<Head>& H, double B_tot, const Opts& o, c
     std::fill(nw.begin(), nw.end(), INF);
     int16_t* ch = choice.data() + (size_t)h * (cap + 1);
     for (size_t k = 0; k < opts[h].size(); ++k) {
-      const Opt& x = opts[h][k];
+      const RateOpt& x = opts[h][k];
       if (x.rate > cap) break;
       for (long long beta = x.rate; beta <= cap; ++beta) {
         double cand = dp[beta - x.rate] + x.D;
@@ -230,7 +226,7 @@ cobra_status exact_dp(const std::vector<Head>& H, double B_tot, const Opts& o, c
   for (int h = n - 1; h >= 0; --h) {
     int k = choice[(size_t)h * (cap + 1) + beta];
     if (k < 0) return COBRA_EBUDGET;
-    const Opt& x = opts[h][k];
+    const RateOpt& x = opts[h][k];
     r[h] = x.r;
     b[h] = x.b;
     D[h] = x.D;
@@ -239,7 +235,67 @@ cobra_status exact_dp(const std::vector<Head>& H, double B_tot, const Opts& o, c
   return COBRA_OK;
 }
 
+// the surrogate's options: every (r, b) of the grid, D from Eq. drb-preview
+cobra_status exact_dp(const std::vector<Head>& H, double B_tot, const Opts& o, const std::vector<int>& grid,
+                      std::vector<int>& r, std::vector<int>& b, std::vector<double>& D) {
+  const int n = (int)H.size();
+  std::vector<std::vector<RateOpt>> opts(n);
+  for (int h = 0; h < n; ++h) {
+    std::vector<RateOpt> all;
+    for (int rr : grid) {
+      if (rr == 0) {
+        all.push_back({0, distortion(H[h], 0, 0), 0, 0});
+        continue;
+      }
+      for (int bb = o.b_min; bb <= o.b_max; ++bb) all.push_back({(long long)rr * bb, distortion(H[h], rr, bb), rr, bb});
+    }
+    opts[h] = unique_by_rate(all);
+  }
+  return dp_over_options(opts, B_tot, r, b, D);
+}
+
 }  // namespace
+
+extern "C" cobra_status cobra_allocate_tables(int n_heads, int d, int n_r, const int* r_list, int n_b,
+                                              const int* b_list, const double* D, double bpd, int* r_out, int* b_out,
+                                              double* dist, long long* rate_bits) {
+  if (n_heads <= 0 || d <= 0 || d > 4096 || n_r <= 0 || n_b <= 0 || !r_list || !b_list || !D || !r_out || !b_out ||
+      !(bpd >= 0.0) || !std::isfinite(bpd))
+    return COBRA_EINVAL;
+  for (int i = 0; i < n_r; ++i)
+    if (r_list[i] < 0 || r_list[i] > d || (i > 0 && r_list[i] <= r_list[i - 1])) return COBRA_EINVAL;
+  for (int j = 0; j < n_b; ++j)
+    if (b_list[j] < 1 || b_list[j] > 16 || (j > 0 && b_list[j] <= b_list[j - 1])) return COBRA_EINVAL;
+  for (long long k = 0; k < (long long)n_heads * n_r * n_b; ++k)
+    if (!std::isfinite(D[k])) return COBRA_EINVAL;
+  std::vector<std::vector<RateOpt>> opts(n_heads);
+  for (int h = 0; h < n_heads; ++h) {
+    std::vector<RateOpt> all;
+    for (int i = 0; i < n_r; ++i) {
+      const double* row = D + ((size_t)h * n_r + i) * n_b;
+      if (r_list[i] == 0) {
+        all.push_back({0, row[0], 0, 0});
+        continue;
+      }
+      for (int j = 0; j < n_b; ++j) all.push_back({(long long)r_list[i] * b_list[j], row[j], r_list[i], b_list[j]});
+    }
+    opts[h] = unique_by_rate(all);
+  }
+  std::vector<int> r(n_heads), b(n_heads);
+  std::vector<double> Dh(n_heads);
+  const double B_tot = (double)((long long)n_heads * d) * bpd;
+  cobra_status st = dp_over_options(opts, B_tot, r, b, Dh);
+  if (st != COBRA_OK) return st;
+  long long used = 0;
+  for (int h = 0; h < n_heads; ++h) {
+    r_out[h] = r[h];
+    b_out[h] = b[h];
+    if (dist) dist[h] = Dh[h];
+    used += (long long)r[h] * b[h];
+  }
+  if (rate_bits) *rate_bits = used;
+  return COBRA_OK;
+}
 
 extern "C" void cobra_alloc_opts_default(cobra_alloc_opts* o) {
   if (!o) return;
