@@ -98,6 +98,24 @@ void cobra_alloc_opts_default(cobra_alloc_opts* o);
 cobra_status cobra_allocate(int n_heads, int d, const double* w, double bpd, const cobra_alloc_opts* opts,
                             int* r, int* b, double* budget, double* dist, long long* rate_bits);
 
+/* App. E "Exact DP over measured distortion", the tables (device, asynchronous on `stream`):
+ * every head's calibration tokens go through the deployed quantizer once per candidate
+ * (r_list[i], b_list[j]) (W = U_r H_r^T with the head's Hadamard signs, Delta = 2 L_b
+ * sigma_bar_r / 2^b rounded to fp32 as cobra_fuse_basis stores it, codes, reconstruction)
+ * and D[h][i][j] = (1/n_tok) sum_t sum_k omega_k (u_k . (x_t - x^_t))^2 is written in fp64,
+ * omega_k = 1 for the MSE objective or sigma_Q,k^2 for attention-KL, so that r = 0 gives
+ * sum_k w_k.  Device inputs, per head h and d = 128: x [n_heads][n_tok][d] fp32 tokens; U
+ * [n_heads][d*d] fp32, column k = u_k in the allocator's order; lam [n_heads][d] fp64
+ * eigenvalues in the same order; omega, mu [n_heads][d] fp32; signs [n_heads][d] int8 (+1/-1).
+ * coords: device workspace of n_heads * n_tok * d floats (overwritten).  Host lists: r_list
+ * (1..65 entries) strictly ascending in [0, 128], b_list (1..16 entries) in [1, 8].  Two
+ * launches; nothing is synchronised.  Errors: EINVAL, EALIGN (4-byte floats, 8-byte
+ * doubles), ECUDA. */
+cobra_status cobra_measure_distortion(int n_heads, int n_tok, const float* x, const float* U, const double* lam,
+                                      const float* omega, const float* mu, const int8_t* signs, int n_r,
+                                      const int* r_list, int n_b, const int* b_list, float* coords, double* D,
+                                      void* stream);
+
 /* App. E "Exact DP over measured distortion": the exact DP of COBRA_ALLOC_EXACT run on
  * explicit per-head distortion tables (e.g. from cobra_measure_distortion) instead of the
  * surrogate.  D: host [n_heads][n_r][n_b] fp64, D[h][i][j] = head h's distortion at

@@ -57,6 +57,8 @@ SIGNATURES = {
     "cobra_alloc_opts_default": (None, [ctypes.POINTER(AllocOpts)]),
     "cobra_allocate": (c_int, [c_int, c_int, P_double, c_double, ctypes.POINTER(AllocOpts), P_int, P_int, P_double,
                                P_double, P_ll]),
+    "cobra_measure_distortion": (c_int, [c_int, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                         c_int, P_int, c_int, P_int, c_void_p, c_void_p, c_void_p]),
     "cobra_allocate_tables": (c_int, [c_int, c_int, c_int, P_int, c_int, P_int, P_double, c_double, P_int, P_int,
                                       P_double, P_ll]),
     "cobra_loading_factor": (c_int, [c_int, P_double]),
@@ -194,6 +196,18 @@ def cobra_allocate_tables(tables, r_list, b_list, bpd: float, d: int = 128):
                                      b.ctypes.data_as(P_int), dist.ctypes.data_as(P_double), ctypes.byref(rate))
     _chk("cobra_allocate_tables", st)
     return dict(r=r, b=b, dist=dist, rate_bits=rate.value)
+
+
+def cobra_measure_distortion(x, U, lam, omega, mu, signs, r_list, b_list, coords, D, stream=None):
+    """Measured distortion tables on the device (App. E); all array arguments are device
+    tensors except the two host lists."""
+    rl, rlp = _np(r_list, np.int32, c_int)
+    bl, blp = _np(b_list, np.int32, c_int)
+    n_heads, n_tok = int(x.shape[0]), int(x.shape[1])
+    st = lib().cobra_measure_distortion(n_heads, n_tok, _ptr(x), _ptr(U), _ptr(lam), _ptr(omega), _ptr(mu),
+                                        _ptr(signs), len(rl), rlp, len(bl), blp, _ptr(coords), _ptr(D),
+                                        _stream(stream))
+    _chk("cobra_measure_distortion", st)
 
 
 def cobra_loading_factor(b: int) -> float:

@@ -14,6 +14,7 @@
 #include "compress_tc.cuh"
 #include "decode.cuh"
 #include "decode_heads.cuh"
+#include "measure.cuh"
 
 using namespace cobra;
 
@@ -587,3 +588,42 @@ extern "C" cobra_status cobra_check(void* stream) {
   }
   return COBRA_OK;
 }
+
+extern "C" cobra_status cobra_measure_distortion(int n_heads, int n_tok, const float* x, const float* U,
+                                                 const double* lam, const float* omega, const float* mu,
+                                                 const int8_t* signs, int n_r, const int* r_list, int n_b,
+                                                 const int* b_list, float* coords, double* D, void* stream) {
+  if (n_heads < 1 || n_heads > 65535 || n_tok < 1 || !x || !U || !lam || !omega || !mu || !signs || !r_list ||
+      !b_list || !coords || !D || n_r < 1 || n_r > kMeasureMaxR || n_b < 1 || n_b > kMeasureMaxB)
+    return COBRA_EINVAL;
+  if (!aligned(x, 4) || !aligned(U, 4) || !aligned(lam, 8) || !aligned(omega, 4) || !aligned(mu, 4) ||
+      !aligned(coords, 4) || !aligned(D, 8))
+    return COBRA_EALIGN;
+  MeasureArgs a{};
+  a.x = x;
+  a.U = U;
+  a.lam = lam;
+  a.omega = omega;
+  a.mu = mu;
+  a.signs = signs;
+  a.coords = coords;
+  a.D = D;
+  a.n_tok = n_tok;
+  a.n_r = n_r;
+  a.n_b = n_b;
+  for (int i = 0; i < n_r; ++i) {
+    if (r_list[i] < 0 || r_list[i] > kD || (i > 0 && r_list[i] <= r_list[i - 1])) return COBRA_EINVAL;
+    a.r[i] = r_list[i];
+  }
+  for (int j = 0; j < n_b; ++j) {
+    if (b_list[j] < 1 || b_list[j] > 8) return COBRA_EINVAL;
+    a.b[j] = b_list[j];
+    if (cobra_loading_factor(b_list[j], &a.L[j]) != COBRA_OK) return COBRA_EINVAL;
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  coords_kernel<<<dim3((unsigned)((n_tok + kCoordTok - 1) / kCoordTok), (unsigned)n_heads), 256, 0, s>>>(a);
+  if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
+  measure_kernel<<<dim3((unsigned)n_r, (unsigned)n_heads), 256, 0, s>>>(a);
+  return launch_status();
+}
+
