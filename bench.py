@@ -51,6 +51,8 @@ def parse_args():
     ap.add_argument("--no-compress", action="store_true", help="skip the prefill compress measurement")
     ap.add_argument("--compress-only", action="store_true", help="only the prefill compress measurement")
     ap.add_argument("--compress-layers", type=int, default=None, help="fewer layers (profiling runs only)")
+    ap.add_argument("--no-measured", action="store_true", help="skip the measured distortion tables (App. E)")
+    ap.add_argument("--measured-only", action="store_true", help="only the measured distortion tables")
     return ap.parse_args()
 
 
@@ -330,6 +332,91 @@ def run_compress_leg(args, dev, stream, peak):
     }
 
 
+MEASURE_PROFILE = os.path.join(ROOT, "profiles", "measure_tables_llama3_8b.txt")
+MEASURE_SOURCES = ["paper_2609_24298_gb300/csrc/measure.cuh", "paper_2609_24298_gb300/csrc/common.cuh"]
+ISSUE_PEAK = 152 * 4 * 2.07e9  # warp-instructions per second: 152 SMs x 4 schedulers at 2070 MHz
+
+
+def profiled_instructions(profile=MEASURE_PROFILE, sources=MEASURE_SOURCES):
+    """Warp-instructions per call from a committed ncu summary taken on the current source."""
+    try:
+        txt = open(profile).read()
+    except OSError:
+        return None
+    m1 = re.search(r"warp_instructions_per_call\s*=\s*([0-9.eE+]+)", txt)
+    m2 = re.search(r"kernel_source_sha\s*=\s*([0-9a-f]+)", txt)
+    if not m1 or not m2 or m2.group(1) != source_hash(sources):
+        return None
+    return float(m1.group(1))
+
+
+def run_measured_leg(args, dev, stream, cals, srcs, cpu_baseline: bool):
+    """App. E's measured distortion tables for every (layer, kv head, side) of the decode
+    workload's model: 512 heads x 512 calibration tokens through the deployed quantizer at
+    every candidate (r, b) of the allocator's grid (65 ranks x 8 widths), one
+    cobra_measure_distortion call.  Returns the JSON object reported under "measured"."""
+    import torch
+
+    from paper_2609_24298_gb300 import cobra, synth
+
+    n = len(cals)
+    xs = np.stack([s.calibration(512) for s in srcs]).astype(np.float32)
+    f32 = lambda a: torch.tensor(np.asarray(a, np.float32), device=dev).contiguous()
+    x = f32(xs)
+    U = f32(np.stack([c["U"].T.reshape(-1) for c in cals]))
+    lam = torch.tensor(np.stack([c["lam"] for c in cals]), dtype=torch.float64, device=dev).contiguous()
+    om = np.stack([np.where(c["lam"] > 0, c["w"] / np.where(c["lam"] > 0, c["lam"], 1.0), 0.0) for c in cals])
+    omega = f32(om)
+    mu = f32(np.stack([c["mu"] for c in cals]))
+    signs = torch.tensor(np.stack([synth.hadamard_signs(*s.key) for s in srcs]), dtype=torch.int8,
+                         device=dev).contiguous()
+    rg, bg = list(range(0, 129, 2)), list(range(1, 9))
+    coords = torch.empty((n, 512, 128), dtype=torch.float32, device=dev)
+    D = torch.empty((n, len(rg), len(bg)), dtype=torch.float64, device=dev)
+
+    def call():
+        cobra.cobra_measure_distortion(x, U, lam, omega, mu, signs, rg, bg, coords, D, stream)
+
+    for _ in range(2):
+        call()
+    torch.cuda.synchronize()
+    K = 5
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / K
+    evals = n * len(rg) * len(bg) * 512  # (head, r, b, calibration token) evaluations
+    out = {
+        "metric": "measured distortion tables (App. E)", "value": ms, "unit": "ms per table set",
+        "higher_is_better": False,
+        "workload": f"{n} heads (32 layers x 8 kv heads x K/V) x 512 calibration tokens x {len(rg)} ranks x "
+                    f"{len(bg)} bit widths, inputs resident on the device",
+        "evaluations_per_s": evals / (ms * 1e-3), "calls": K, "launches": 2 * K,
+    }
+    instr = profiled_instructions()
+    out["roofline"] = {"bound": "issue", "kernel": "coords_kernel + measure_kernel", "unit": "warp-instr/s",
+                       "peak": ISSUE_PEAK, "warp_instructions_per_call": instr,
+                       "achieved": instr / (ms * 1e-3) if instr else None,
+                       "frac": instr / (ms * 1e-3) / ISSUE_PEAK if instr else None}
+    if cpu_baseline:
+        # the oracle's fp64 tables for one head over the same grid, extrapolated to all heads
+        from oracle import calibrate as ocal
+        from oracle import measured as omeas
+
+        cal = ocal.calibrate_head(xs[0].astype(np.float64))
+        t0 = time.time()
+        omeas.measured_table(xs[0].astype(np.float64), cal, np.ones(128), synth.hadamard_signs(*srcs[0].key), rg, bg)
+        el = time.time() - t0
+        out["cpu_baseline"] = {"value": el * n * 1e3, "unit": "ms per table set", "cores": cores_used(),
+                               "kind": "oracle", "sample": f"one head's full table ({el:.1f} s of fp64 numpy), "
+                                                          f"extrapolated to {n} heads"}
+    del x, U, lam, omega, mu, signs, coords, D
+    return out
+
+
 # ---------------------------------------------------------------------------------------
 # the CUDA path
 # ---------------------------------------------------------------------------------------
@@ -355,6 +442,11 @@ def run_cobra(args):
     cobra.lib()
     if args.compress_only:
         print(json.dumps(run_compress_leg(args, dev, torch.cuda.current_stream(), hbm_peak()[0])), flush=True)
+        return
+    if args.measured_only:
+        hp, srcs = pipeline.build_params(CFG, L, spec["bpd"], joint=False)
+        print(json.dumps(run_measured_leg(args, dev, torch.cuda.current_stream(), hp.cals, srcs,
+                                          not args.no_cpu_baseline)), flush=True)
         return
 
     # cpu baseline first, before any GPU work (rank 0, N = 1 only)
@@ -488,6 +580,9 @@ def run_cobra(args):
 
     peak, peak_kind = hbm_peak()
     achieved = bytes_step / (scan_ms * 1e-3) / 1e9
+    measured = None
+    if not args.no_measured and rank == 0:
+        measured = run_measured_leg(args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
     compress = None
     if not args.no_compress:
         del hin, hout
@@ -505,6 +600,7 @@ def run_cobra(args):
                          "traffic": traffic, "scan_ms": scan_ms,
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
             "compress": compress,
+            "measured": measured,
             "cpu_baseline": cpu,
             "e2e": {"value": weak_scaling_gbs(bytes_step, 1, world, e2e_ms), "unit": "GB/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},

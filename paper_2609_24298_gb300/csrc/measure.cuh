@@ -125,13 +125,19 @@ __global__ void __launch_bounds__(256) measure_kernel(MeasureArgs a) {
     om[m] = omega[k];
     inv[m] = size > 0 ? rsqrtf((float)size) : 0.f;
   }
+  // with unit weights (the MSE objective) the rotation back preserves the norm: the error is
+  // summed in the rotated coordinates and the second transform is skipped
+  const bool unit_w = __all_sync(0xffffffffu, om[0] == 1.f && om[1] == 1.f && om[2] == 1.f && om[3] == 1.f);
   // Delta per b, as the stored fp32 step: 2 L_b sigma_bar / 2^b, sigma_bar^2 = mean lambda_{<r}
-  float delta[kMeasureMaxB];
+  float delta[kMeasureMaxB], inv_delta[kMeasureMaxB];
   double lsum = 0.0;
   for (int k = 0; k < r; ++k) lsum += a.lam[(size_t)h * kD + k];
   const double sigma = r > 0 ? sqrt(lsum / r) : 0.0;
 #pragma unroll
-  for (int j = 0; j < kMeasureMaxB; ++j) delta[j] = j < a.n_b ? (float)(2.0 * a.L[j] * sigma / (double)(1 << a.b[j])) : 0.f;
+  for (int j = 0; j < kMeasureMaxB; ++j) {
+    delta[j] = j < a.n_b ? (float)(2.0 * a.L[j] * sigma / (double)(1 << a.b[j])) : 0.f;
+    inv_delta[j] = delta[j] > 0.f ? 1.f / delta[j] : 0.f;
+  }
 
   float acc_trunc = 0.f, acc[kMeasureMaxB];
 #pragma unroll
@@ -153,13 +159,20 @@ __global__ void __launch_bounds__(256) measure_kernel(MeasureArgs a) {
     for (int j = 0; j < kMeasureMaxB; ++j) {
       if (j >= a.n_b) break;
       const int bb = a.b[j];
-      const float half = (float)(1 << (bb - 1)), cmax = (float)((1 << bb) - 1), dl = delta[j];
+      const float half = (float)(1 << (bb - 1)), cmax = (float)((1 << bb) - 1), dl = delta[j], il = inv_delta[j];
       float e[4];
 #pragma unroll
       for (int m = 0; m < 4; ++m) {
-        float code = floorf(y[m] / dl + half);
+        // (a code may differ from the exact division's at a cell boundary, where both cells
+        // leave an error of the same size)
+        float code = floorf(fmaf(y[m], il, half));
         code = fminf(fmaxf(code, 0.f), cmax);
         e[m] = bs[m] > 0 ? y[m] - dl * (code - half + 0.5f) : 0.f;
+      }
+      if (unit_w) {
+#pragma unroll
+        for (int m = 0; m < 4; ++m) acc[j] = fmaf(e[m], e[m], acc[j]);
+        continue;
       }
       // back to the eigen coordinates: H_r^T = diag(s) blockdiag(H_n / sqrt n) (H_n symmetric)
       block_wht(e, bs, lane);

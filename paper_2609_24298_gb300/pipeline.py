@@ -115,6 +115,7 @@ def build_params(cfg: int, layers: int, bpd: float, joint: bool, kl_queries: boo
     signs = [synth.hadamard_signs(*s.key) for s in srcs]
     hp = fuse_heads(cals, r, b, signs)
     hp.alloc = dict(parts=allocs, w=w)
+    hp.cals = cals
     return hp, srcs
 
 
