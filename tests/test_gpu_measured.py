@@ -106,3 +106,35 @@ def test_full_candidate_grid_and_dp():
             alt = sum(want[h][rg.index(int(a["r"][h]))][bg.index(int(a["b"][h])) if a["r"][h] else 0]
                       for h in range(len(hs)))
             assert alt <= tot * (1 + 1e-3)
+
+
+def test_measured_allocation_end_to_end():
+    """App. E's allocator on the tiny model (1 layer x 8 kv heads, K with attention-KL weights,
+    V with MSE weights, 2 bpd): the library's calibration, device tables and table DP give the
+    oracle's allocation from the oracle's calibration and tables (or an equally good
+    near-tie), and a cache built with that allocation decodes within the decode tolerance."""
+    from paper_2609_24298_gb300 import pipeline
+
+    from .gpu_util import oracle_calibrations
+    from .test_gpu_fullsize import run_workload
+
+    cfg, bpd = 1, 2.0
+    cals, srcs = oracle_calibrations(cfg, 1)
+    spec = synth.CONFIGS[cfg]
+    qs = [synth.calibration_queries(cfg, s.key[1], s.key[2], spec["q_heads"] // spec["kv_heads"], 512, spec["alpha"])
+          if s.key[3] == 0 else None for s in srcs]
+    lib_cals = pipeline.calibrate_heads([s.calibration(512) for s in srcs], qs)
+    r, b = pipeline.measured_allocation(lib_cals, srcs, bpd, device=DEV)
+    rg, bg = om.default_grids()
+    n = len(cals) // 2
+    for side in (0, 1):
+        part = slice(side * n, (side + 1) * n)
+        tabs = [om.measured_table(s.calibration(512), c, om.error_weights(c, q), synth.hadamard_signs(*s.key), rg, bg)
+                for c, s, q in zip(cals[part], srcs[part], qs[part])]
+        ro, bo, _, tot = om.exact_dp_tables(tabs, rg, bg, n * 128 * bpd)
+        if list(r[part]) != ro or list(b[part]) != bo:
+            alt = sum(t[rg.index(int(rr))][bg.index(int(bb)) if rr else 0] for t, rr, bb in zip(tabs, r[part], b[part]))
+            assert alt <= tot * (1 + 1e-3)
+    params = [ocal.head_params(c, int(rr), int(bb) if rr else 1, synth.hadamard_signs(*s.key))
+              for c, s, rr, bb in zip(cals, srcs, r, b)]
+    run_workload(cfg, 1, params, srcs, [2048], [(0, h, 0) for h in range(8)])
