@@ -52,6 +52,9 @@ def parse_args():
     ap.add_argument("--compress-only", action="store_true", help="only the prefill compress measurement")
     ap.add_argument("--compress-layers", type=int, default=None, help="fewer layers (profiling runs only)")
     ap.add_argument("--no-measured", action="store_true", help="skip the measured distortion tables (App. E)")
+    ap.add_argument("--k-bpd", type=float, default=None, help="K rate of a K+V split (default: the workload's)")
+    ap.add_argument("--v-bpd", type=float, default=None, help="V rate of a K+V split (default: the workload's)")
+    ap.add_argument("--v-uniform", action="store_true", help="V by the uniform per-head budget (App. vside)")
     ap.add_argument("--measured-only", action="store_true", help="only the measured distortion tables")
     return ap.parse_args()
 
@@ -258,6 +261,14 @@ def workload_config(spec):
             "l2": "inputs larger than L2 (packed cache of about 2 GiB re-read every step)"}
 
 
+def split_config(args):
+    """The K+V split of a non-default run (Sec. 5 "Joint K+V compression", App. vside)."""
+    if args.k_bpd is None and args.v_bpd is None and not args.v_uniform:
+        return {}
+    return {"workload": "llama3-8b-shaped decode step with a K+V rate split", "k_bpd": args.k_bpd,
+            "v_bpd": args.v_bpd, "v_allocation": "uniform per head" if args.v_uniform else "damped"}
+
+
 # ---------------------------------------------------------------------------------------
 # prefill compress (the tensor-core projection path)
 # ---------------------------------------------------------------------------------------
@@ -457,7 +468,9 @@ def run_cobra(args):
                "sample": f"{n} (seq, layer, kv-head) decode steps over {T} tokens with K and V at r={SAMPLE_R}, "
                          f"b={SAMPLE_B} incl. append-compress ({el:.1f} s of fp64 numpy)"}
 
-    hp, srcs = pipeline.build_params(CFG, L, spec["bpd"], joint=False)
+    k_bpd = args.k_bpd if args.k_bpd is not None else spec["bpd"]
+    v_opts = cobra.alloc_opts(mode=2) if args.v_uniform else None  # 2: COBRA_ALLOC_UNIFORM
+    hp, srcs = pipeline.build_params(CFG, L, k_bpd, joint=False, v_bpd=args.v_bpd, v_opts=v_opts)
     rows = -(-T // 128)
     wl = pipeline.Workload(cfg=CFG, layers=L, kv=H, group=G, seqs=S, tokens=np.full(S, T - 1, np.int64),
                            bpd=spec["bpd"], joint=False, rows_per_seq=rows)
@@ -593,7 +606,7 @@ def run_cobra(args):
             "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": K, "warmup": args.warmup,
             "ms_per_step": total_ms / K, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "fp16-mma/fp32-acc on 1-8 bit codes", "data": "synthetic", "impl": "cobra",
-            "config": workload_config(spec) | {"parallelism": f"replicas x{world}", "layers": L,
+            "config": workload_config(spec) | split_config(args) | {"parallelism": f"replicas x{world}", "layers": L,
                                                "packed_bytes_per_step": bytes_step},
             "roofline": {"bound": "hbm", "kernel": "decode_kernel (rank-space scan)", "achieved": achieved,
                          "peak": peak, "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,

@@ -86,9 +86,12 @@ class Workload:
         return self.layers * self.kv
 
 
-def build_params(cfg: int, layers: int, bpd: float, joint: bool, kl_queries: bool = True, alloc_opts=None):
+def build_params(cfg: int, layers: int, bpd: float, joint: bool, kl_queries: bool = True, alloc_opts=None,
+                 v_bpd: float | None = None, v_opts=None):
     """Calibrate every (layer, kv head, side) of a config on 512 calibration tokens, allocate
-    (K and V separately, or jointly over both sides with MSE weights), fuse the bases."""
+    (K and V separately, or jointly over both sides with MSE weights), fuse the bases.  With
+    v_bpd the V side gets its own rate (the K+V split of Sec. 5, "Joint K+V compression") and
+    v_opts its own allocator options (e.g. the uniform per-head budget of App. vside)."""
     spec = synth.CONFIGS[cfg]
     H = spec["kv_heads"]
     G = spec["q_heads"] // H
@@ -109,7 +112,7 @@ def build_params(cfg: int, layers: int, bpd: float, joint: bool, kl_queries: boo
         allocs = [res]
     else:
         rk = cobra.cobra_allocate(w[:n], bpd, alloc_opts)
-        rv = cobra.cobra_allocate(w[n:], bpd, alloc_opts)
+        rv = cobra.cobra_allocate(w[n:], bpd if v_bpd is None else v_bpd, alloc_opts if v_opts is None else v_opts)
         r, b = np.concatenate([rk["r"], rv["r"]]), np.concatenate([rk["b"], rv["b"]])
         allocs = [rk, rv]
     signs = [synth.hadamard_signs(*s.key) for s in srcs]

@@ -15,6 +15,8 @@ import numpy as np
 import pytest
 import torch
 
+from oracle import allocator as oal
+from oracle import calibrate as ocal
 from oracle import compress as ocomp
 from oracle import layout as olay
 from paper_2609_24298_gb300 import cobra, pipeline, synth
@@ -213,3 +215,20 @@ def _sweep_calibrations(layers):
     if layers not in _SWEEP:
         _SWEEP[layers] = oracle_calibrations(5, layers)
     return _SWEEP[layers]
+
+
+@pytest.mark.parametrize("k_bpd,v_bpd", [(1.5, 0.5), (0.5, 1.5)])
+def test_kv_split_with_uniform_v(k_bpd, v_bpd):
+    """The K+V protocol of Sec. 5 ("Joint K+V compression") and App. vside: a total of 2 bpd
+    split between the sides, K allocated by the damped allocator on attention-KL weights and V
+    by the uniform per-head budget (C1 only); Llama-3-8B shape (batch 8 x 32768 tokens), 4 of
+    its 32 layers (the layers are independent and shaped alike)."""
+    cals, srcs = oracle_calibrations(2, 4)
+    n = len(cals) // 2
+    w = np.stack([c["w"] for c in cals])
+    k = oal.allocate(w[:n], k_bpd)
+    v = oal.allocate(w[n:], v_bpd, oal.Opts(mode=oal.MODE_UNIFORM))
+    r, b = np.concatenate([k["r"], v["r"]]), np.concatenate([k["b"], v["b"]])
+    params = [ocal.head_params(c, int(rr), int(bb) if rr else 1, synth.hadamard_signs(*s.key))
+              for c, s, rr, bb in zip(cals, srcs, r, b)]
+    run_workload(2, 4, params, srcs, [32768] * 8, [(0, 0, 0), (1, 5, 3), (3, 7, 7)])
