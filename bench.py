@@ -56,6 +56,8 @@ def parse_args():
     ap.add_argument("--v-bpd", type=float, default=None, help="V rate of a K+V split (default: the workload's)")
     ap.add_argument("--v-uniform", action="store_true", help="V by the uniform per-head budget (App. vside)")
     ap.add_argument("--measured-only", action="store_true", help="only the measured distortion tables")
+    ap.add_argument("--no-calibration", action="store_true", help="skip the device calibration leg")
+    ap.add_argument("--calibration-only", action="store_true", help="only the device calibration leg")
     return ap.parse_args()
 
 
@@ -361,6 +363,90 @@ def profiled_instructions(profile=MEASURE_PROFILE, sources=MEASURE_SOURCES):
     return float(m1.group(1))
 
 
+CALIB_PROFILE = os.path.join(ROOT, "profiles", "calibrate_heads_llama3_8b.txt")
+CALIB_SOURCES = ["paper_2609_24298_gb300/csrc/calib.cuh", "paper_2609_24298_gb300/csrc/common.cuh"]
+FP64_NOMINAL_TFLOPS = 1.25  # GB300's fp64 rate (nominal; no measured figure on this machine)
+
+
+def profiled_value(key, profile, sources):
+    """A per-call figure from a committed ncu summary taken on the current source."""
+    try:
+        txt = open(profile).read()
+    except OSError:
+        return None
+    m1 = re.search(key + r"\s*=\s*([0-9.eE+]+)", txt)
+    m2 = re.search(r"kernel_source_sha\s*=\s*([0-9a-f]+)", txt)
+    if not m1 or not m2 or m2.group(1) != source_hash(sources):
+        return None
+    return float(m1.group(1))
+
+
+def run_calibration_leg(args, dev, stream, srcs, cpu_baseline: bool):
+    """Table alg:kvrobin steps 1-2 for the decode workload's model on the device: 512 heads x
+    512 calibration vectors (the 256 K heads with their groups' 2048 calibration queries,
+    attention-KL weights; the 256 V heads with MSE weights), two cobra_calibrate_heads calls.
+    Returns the JSON object reported under "calibration"."""
+    import torch
+
+    from paper_2609_24298_gb300 import cobra, pipeline, synth
+
+    spec = synth.CONFIGS[CFG]
+    G = spec["q_heads"] // spec["kv_heads"]
+    xs = [s.calibration(512) for s in srcs]
+    qs = [synth.calibration_queries(CFG, s.key[1], s.key[2], G, 512, spec["alpha"]) if s.key[3] == 0 else None
+          for s in srcs]
+    calls = []
+    for kl in (True, False):
+        idx = [i for i, q in enumerate(qs) if (q is not None) == kl]
+        x = torch.tensor(np.stack([np.asarray(xs[i], np.float32) for i in idx]), device=dev).contiguous()
+        q = torch.tensor(np.stack([np.asarray(qs[i], np.float32).reshape(-1, 128) for i in idx]),
+                         device=dev).contiguous() if kl else None
+        outs = [torch.empty((len(idx), n), dtype=torch.float64, device=dev) for n in (128, 128, 128 * 128, 128)]
+        calls.append((x, q, outs))
+
+    def call():
+        for x, q, (mu, lam, U, w) in calls:
+            cobra.cobra_calibrate_heads(x, q, mu, lam, U, w, stream)
+
+    call()
+    torch.cuda.synchronize()
+    K = 3
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / K
+    t0 = time.time()
+    pipeline.calibrate_heads(xs, qs)
+    host_ms = (time.time() - t0) * 1e3
+    flops = profiled_value("fp64_flops_per_call", CALIB_PROFILE, CALIB_SOURCES)
+    out = {
+        "metric": "calibration steps 1-2 (covariance, eigen-decomposition, KL weights and order)", "value": ms,
+        "unit": "ms for all heads", "higher_is_better": False,
+        "workload": f"{len(srcs)} heads (32 layers x 8 kv heads x K/V) x 512 calibration vectors; K heads with "
+                    f"{G * 512} calibration queries each",
+        "calls": K, "launches": 2 * K,
+        "host_library_ms": host_ms, "host_library_threads": pipeline._threads(),
+        "roofline": {"bound": "fp64", "kernel": "calib_kernel", "unit": "TFLOP/s", "peak": FP64_NOMINAL_TFLOPS,
+                     "peak_kind": "nominal", "fp64_flops_per_call": flops,
+                     "achieved": flops / (ms * 1e-3) / 1e12 if flops else None,
+                     "frac": flops / (ms * 1e-3) / 1e12 / FP64_NOMINAL_TFLOPS if flops else None},
+    }
+    if cpu_baseline:
+        from oracle import calibrate as ocal
+
+        t0 = time.time()
+        ocal.calibrate_head(np.asarray(xs[0], np.float64), qs[0])
+        el = time.time() - t0
+        out["cpu_baseline"] = {"value": el * len(srcs) * 1e3, "unit": "ms for all heads", "cores": cores_used(),
+                               "kind": "oracle", "sample": f"one K head ({el * 1e3:.1f} ms of fp64 numpy), "
+                                                          f"extrapolated to {len(srcs)} heads"}
+    del calls
+    return out
+
+
 def run_measured_leg(args, dev, stream, cals, srcs, cpu_baseline: bool):
     """App. E's measured distortion tables for every (layer, kv head, side) of the decode
     workload's model: 512 heads x 512 calibration tokens through the deployed quantizer at
@@ -454,6 +540,11 @@ def run_cobra(args):
     if args.compress_only:
         print(json.dumps(run_compress_leg(args, dev, torch.cuda.current_stream(), hbm_peak()[0])), flush=True)
         return
+    if args.calibration_only:
+        srcs = [synth.HeadSource(CFG, l, h, side, spec["alpha"]) for side in (0, 1) for l in range(L) for h in range(H)]
+        print(json.dumps(run_calibration_leg(args, dev, torch.cuda.current_stream(), srcs,
+                                             not args.no_cpu_baseline)), flush=True)
+        return
     if args.measured_only:
         hp, srcs = pipeline.build_params(CFG, L, spec["bpd"], joint=False)
         print(json.dumps(run_measured_leg(args, dev, torch.cuda.current_stream(), hp.cals, srcs,
@@ -469,7 +560,7 @@ def run_cobra(args):
                          f"b={SAMPLE_B} incl. append-compress ({el:.1f} s of fp64 numpy)"}
 
     k_bpd = args.k_bpd if args.k_bpd is not None else spec["bpd"]
-    v_opts = cobra.alloc_opts(mode=2) if args.v_uniform else None  # 2: COBRA_ALLOC_UNIFORM
+    v_opts = cobra.alloc_opts(mode=cobra.ALLOC_UNIFORM) if args.v_uniform else None
     hp, srcs = pipeline.build_params(CFG, L, k_bpd, joint=False, v_bpd=args.v_bpd, v_opts=v_opts)
     rows = -(-T // 128)
     wl = pipeline.Workload(cfg=CFG, layers=L, kv=H, group=G, seqs=S, tokens=np.full(S, T - 1, np.int64),
@@ -593,6 +684,9 @@ def run_cobra(args):
 
     peak, peak_kind = hbm_peak()
     achieved = bytes_step / (scan_ms * 1e-3) / 1e9
+    calibration = None
+    if not args.no_calibration and rank == 0:
+        calibration = run_calibration_leg(args, dev, stream, srcs, not args.no_cpu_baseline and world == 1)
     measured = None
     if not args.no_measured and rank == 0:
         measured = run_measured_leg(args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
@@ -614,6 +708,7 @@ def run_cobra(args):
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
             "compress": compress,
             "measured": measured,
+            "calibration": calibration,
             "cpu_baseline": cpu,
             "e2e": {"value": weak_scaling_gbs(bytes_step, 1, world, e2e_ms), "unit": "GB/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},

@@ -98,6 +98,19 @@ void cobra_alloc_opts_default(cobra_alloc_opts* o);
 cobra_status cobra_allocate(int n_heads, int d, const double* w, double bpd, const cobra_alloc_opts* opts,
                             int* r, int* b, double* budget, double* dist, long long* rate_bits);
 
+/* Table alg:kvrobin steps 1-2 on the device for many heads at once (one CTA per head, fp64):
+ * the same quantities as cobra_calibrate_head - mean, centred (1/N) covariance, its
+ * eigen-decomposition (parallel cyclic Jacobi), eigenvalues descending with each
+ * eigenvector's largest-magnitude component positive, and with calibration queries the
+ * attention-KL weights w_i = sigma_Q,i^2 lambda_i and the stable reorder by w descending
+ * (without: w = lambda).  Device inputs: x [n_heads][n_tok][128] fp32 calibration vectors;
+ * q [n_heads][n_q][128] fp32 queries of each head's group (n_q = 0 and q = NULL for the MSE
+ * objective).  Device outputs (fp64): mu, lam, w [n_heads][128]; U [n_heads][128 * 128] with
+ * U[h][j * 128 + i] = component i of direction j (allocator order).  One launch, nothing is
+ * synchronised.  Errors: EINVAL, EALIGN (4-byte floats, 8-byte doubles), ECUDA. */
+cobra_status cobra_calibrate_heads(int n_heads, int n_tok, const float* x, int n_q, const float* q, double* mu,
+                                   double* lam, double* U, double* w, void* stream);
+
 /* App. E "Exact DP over measured distortion", the tables (device, asynchronous on `stream`):
  * every head's calibration tokens go through the deployed quantizer once per candidate
  * (r_list[i], b_list[j]) (W = U_r H_r^T with the head's Hadamard signs, Delta = 2 L_b

@@ -57,6 +57,8 @@ SIGNATURES = {
     "cobra_alloc_opts_default": (None, [ctypes.POINTER(AllocOpts)]),
     "cobra_allocate": (c_int, [c_int, c_int, P_double, c_double, ctypes.POINTER(AllocOpts), P_int, P_int, P_double,
                                P_double, P_ll]),
+    "cobra_calibrate_heads": (c_int, [c_int, c_int, c_void_p, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                      c_void_p]),
     "cobra_measure_distortion": (c_int, [c_int, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
                                          c_int, P_int, c_int, P_int, c_void_p, c_void_p, c_void_p]),
     "cobra_allocate_tables": (c_int, [c_int, c_int, c_int, P_int, c_int, P_int, P_double, c_double, P_int, P_int,
@@ -196,6 +198,16 @@ def cobra_allocate_tables(tables, r_list, b_list, bpd: float, d: int = 128):
                                      b.ctypes.data_as(P_int), dist.ctypes.data_as(P_double), ctypes.byref(rate))
     _chk("cobra_allocate_tables", st)
     return dict(r=r, b=b, dist=dist, rate_bits=rate.value)
+
+
+def cobra_calibrate_heads(x, q, mu, lam, U, w, stream=None):
+    """Device calibration of many heads (steps 1-2); x [n][n_tok][128], q [n][n_q][128] or
+    None; outputs are device fp64 tensors mu, lam, w [n][128] and U [n][128 * 128]."""
+    n_heads, n_tok = int(x.shape[0]), int(x.shape[1])
+    n_q = int(q.shape[1]) if q is not None else 0
+    st = lib().cobra_calibrate_heads(n_heads, n_tok, _ptr(x), n_q, _ptr(q), _ptr(mu), _ptr(lam), _ptr(U), _ptr(w),
+                                     _stream(stream))
+    _chk("cobra_calibrate_heads", st)
 
 
 def cobra_measure_distortion(x, U, lam, omega, mu, signs, r_list, b_list, coords, D, stream=None):

@@ -15,6 +15,7 @@
 #include "decode.cuh"
 #include "decode_heads.cuh"
 #include "measure.cuh"
+#include "calib.cuh"
 
 using namespace cobra;
 
@@ -624,6 +625,34 @@ extern "C" cobra_status cobra_measure_distortion(int n_heads, int n_tok, const f
   coords_kernel<<<dim3((unsigned)((n_tok + kCoordTok - 1) / kCoordTok), (unsigned)n_heads), 256, 0, s>>>(a);
   if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
   measure_kernel<<<dim3((unsigned)n_r, (unsigned)n_heads), 256, 0, s>>>(a);
+  return launch_status();
+}
+
+extern "C" cobra_status cobra_calibrate_heads(int n_heads, int n_tok, const float* x, int n_q, const float* q,
+                                              double* mu, double* lam, double* U, double* w, void* stream) {
+  if (n_heads < 1 || n_heads > 0x7fffffff || n_tok < 1 || !x || !mu || !lam || !U || !w || n_q < 0 ||
+      (n_q > 0 && !q))
+    return COBRA_EINVAL;
+  if (!aligned(x, 4) || (q && !aligned(q, 4)) || !aligned(mu, 8) || !aligned(lam, 8) || !aligned(U, 8) ||
+      !aligned(w, 8))
+    return COBRA_EALIGN;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(calib_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)calib_smem_bytes()) !=
+        cudaSuccess)
+      return COBRA_ECUDA;
+    attr = true;
+  }
+  CalibArgs a{};
+  a.x = x;
+  a.q = n_q > 0 ? q : nullptr;
+  a.mu = mu;
+  a.lam = lam;
+  a.U = U;
+  a.w = w;
+  a.n_tok = n_tok;
+  a.n_q = n_q;
+  calib_kernel<<<(unsigned)n_heads, kCalThreads, calib_smem_bytes(), (cudaStream_t)stream>>>(a);
   return launch_status();
 }
 

@@ -122,6 +122,32 @@ def build_params(cfg: int, layers: int, bpd: float, joint: bool, kl_queries: boo
     return hp, srcs
 
 
+def calibrate_heads_device(xs, qs=None, device="cuda"):
+    """Steps 1-2 for many heads on the device (cobra_calibrate_heads): the heads with
+    calibration queries (attention-KL weights) in one launch, the others (MSE) in another.
+    Returns the same dicts as calibrate_heads (U[:, j] = direction j)."""
+    qs = qs if qs is not None else [None] * len(xs)
+    out = [None] * len(xs)
+    for kl in (True, False):
+        idx = [i for i, q in enumerate(qs) if (q is not None) == kl]
+        if not idx:
+            continue
+        x = torch.tensor(np.stack([np.asarray(xs[i], np.float32) for i in idx]), device=device).contiguous()
+        q = None
+        if kl:
+            q = torch.tensor(np.stack([np.asarray(qs[i], np.float32).reshape(-1, D) for i in idx]),
+                             device=device).contiguous()
+        n = len(idx)
+        f64 = lambda *shape: torch.empty(shape, dtype=torch.float64, device=device)
+        mu, lam, U, w = f64(n, D), f64(n, D), f64(n, D * D), f64(n, D)
+        cobra.cobra_calibrate_heads(x, q, mu, lam, U, w)
+        torch.cuda.synchronize()
+        mu, lam, U, w = mu.cpu().numpy(), lam.cpu().numpy(), U.cpu().numpy(), w.cpu().numpy()
+        for k, i in enumerate(idx):
+            out[i] = dict(mu=mu[k], lam=lam[k], U=U[k].reshape(D, D).T.copy(), w=w[k])
+    return out
+
+
 def error_weights(cal) -> np.ndarray:
     """omega_k = w_k / lambda_k: 1 for the MSE objective, sigma_Q,k^2 for attention-KL (0 on a
     direction without variance)."""
