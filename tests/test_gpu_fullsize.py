@@ -9,8 +9,8 @@ attend over identical codes: a legitimate boundary flip on a heavily weighted to
 the output by far more than the decode tolerance), and decode runs in the launch
 configuration the benchmark times (query projection, scan, combine on one stream) over the
 whole cache; sampled outputs must be within max relative error 2e-3 of the oracle's attention.
-The single-call entry points (decode attention; the decode step with both appends) must
-reproduce the staged calls bit for bit."""
+The single-call entry points (decode attention; the decode step with both appends, on device
+buffers and on pinned host buffers) must reproduce the staged calls bit for bit."""
 import numpy as np
 import pytest
 import torch
@@ -109,6 +109,7 @@ def run_workload(cfg, layers, params, srcs, lens, samples, paged=False, seed=5):
     block, cache, pt = wl.dev.block, wl.dev.cache, wl.page_table
     stream = torch.cuda.current_stream()
     before = cache.clone()
+    pre = cache.clone()
     cobra.cobra_append(block, adesc[0], xk, pos, cache, pt, stream)
     cobra.cobra_append(block, adesc[1], xv, pos, cache, pt, stream)
     torch.cuda.synchronize()
@@ -121,11 +122,20 @@ def run_workload(cfg, layers, params, srcs, lens, samples, paged=False, seed=5):
                             nws, stream)
     staged_out = torch.full_like(step_out, float("nan"))
     cobra.cobra_decode_attn(block, desc, info, q, cache, lens_d, pt, staged_out, ws, nws, stream)
+    # and on pinned host buffers: the kernels read the tokens and queries from host memory and
+    # write the output there (coherent NVLink-C2C), with the same result
+    host_cache = pre.clone()
+    host_out = torch.full((L, S, H * G, D), float("nan"), dtype=torch.float32).pin_memory()
+    hk_, hv_, hq_ = xk.cpu().pin_memory(), xv.cpu().pin_memory(), q.cpu().pin_memory()
+    cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], hk_, hv_, pos, hq_, host_cache, lens_d, pt, host_out,
+                            ws, nws, stream)
     torch.cuda.synchronize()
     assert cobra.cobra_check(stream) == cobra.COBRA_OK
     assert torch.equal(before, cache)
+    assert torch.equal(host_cache, cache)
     assert torch.equal(step_out, staged_out)
-    del before, step_out, staged_out
+    assert torch.equal(host_out, staged_out.cpu())
+    del before, step_out, staged_out, host_cache, pre
 
     # compress + append parity on the sampled heads, then the oracle's rows in their place
     hk, hv = xk.float().cpu().numpy(), xv.float().cpu().numpy()
