@@ -70,3 +70,35 @@ def test_table_argument_checks():
     with pytest.raises(cobra.CobraError) as e:
         cobra.cobra_allocate_tables(t, [0, 9], [1, 2], 1.0, 8)  # r > d
     assert e.value.status == cobra.COBRA_EINVAL
+
+
+def test_device_entry_points_check_arguments_before_the_gpu():
+    # cobra_measure_distortion and cobra_calibrate_heads validate sizes, lists and alignment on
+    # the host and return before any launch (fake device addresses are never touched)
+    L = cobra.lib()
+    import ctypes
+
+    def measure(n_heads=1, n_tok=4, r=(0, 2), b=(1, 2), x=256, D=256):
+        rl = (ctypes.c_int * len(r))(*r)
+        bl = (ctypes.c_int * len(b))(*b)
+        return L.cobra_measure_distortion(n_heads, n_tok, x, 256, 256, 256, 256, 256, len(r), rl, len(b), bl, 256, D,
+                                          None)
+
+    assert measure(r=()) == cobra.COBRA_EINVAL
+    assert measure(r=tuple(range(0, 132, 2))) == cobra.COBRA_EINVAL  # 66 ranks
+    assert measure(r=(4, 2)) == cobra.COBRA_EINVAL  # not ascending
+    assert measure(r=(0, 130)) == cobra.COBRA_EINVAL  # r > 128
+    assert measure(b=(0,)) == cobra.COBRA_EINVAL
+    assert measure(b=(9,)) == cobra.COBRA_EINVAL
+    assert measure(n_tok=0) == cobra.COBRA_EINVAL
+    assert measure(x=258) == cobra.COBRA_EALIGN
+    assert measure(D=260) == cobra.COBRA_EALIGN
+
+    def calib(n_heads=1, n_tok=4, n_q=0, q=None, x=256, mu=256):
+        return L.cobra_calibrate_heads(n_heads, n_tok, x, n_q, q, mu, 256, 256, 256, None)
+
+    assert calib(n_tok=0) == cobra.COBRA_EINVAL
+    assert calib(n_heads=0) == cobra.COBRA_EINVAL
+    assert calib(n_q=3, q=None) == cobra.COBRA_EINVAL
+    assert calib(x=258) == cobra.COBRA_EALIGN
+    assert calib(mu=260) == cobra.COBRA_EALIGN
