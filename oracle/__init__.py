@@ -16,6 +16,7 @@ Modules
   calibrate  centred covariance, eigenbasis, attention-KL weights and reordering, basis fusion
   layout     the packed code-row layout (bit position of every code)
   attention  dequantise-on-read decode attention, plain definition and rank-space algebra
+  rope       decode with the rotary embedding applied to the reconstructed keys and the query
   compress   per-token projection + quantisation (Table alg:kvrobin step 7)
 
 Parity status: the damped C2 update is a heuristic with no optimality guarantee
