@@ -329,6 +329,39 @@ cobra_status cobra_decode_step(const void* params, const cobra_decode_desc* desc
                                const int* page_table, float* out, void* workspace, size_t ws_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------------------
+ * Decode attention for models with the rotary position embedding (RoPE).  Sec. 5 ("Scope")
+ * and App. "Post-RoPE experiments": K is compressed before the rotation, so the model's
+ * attention turns every reconstructed key to its own position and the query to its position:
+ *   p_t = softmax_t(R(p_s) q . R(t) K^_t / sqrt(d)),  o = sum_t p_t V^_t   (V is not rotated),
+ * R(x) turning channel pair (j, j + 64) by the angle x * theta^(-2j/128) (the rotate-half
+ * form of Llama-3, Mistral and Qwen), key t of a sequence at position t.  The keys are rebuilt
+ * from their codes in the 128-dimensional space on the tensor cores (the rotation differs per
+ * token, so they cannot be folded into one projected query as cobra_decode_attn does).
+ * ------------------------------------------------------------------------------------- */
+
+/* Bytes of the angle table for positions 0 .. max_pos - 1 (1 <= max_pos <= 2^22, else
+ * COBRA_EINVAL): 128 floats per position multiple of 16, plus 16 rows for positions 0..15. */
+cobra_status cobra_rope_table_bytes(int max_pos, size_t* bytes);
+
+/* Fill the angle table (device, 16-byte aligned, >= cobra_rope_table_bytes) for base theta
+ * (> 0; 500000 for Llama-3): cos and sin of x * theta^(-2j/128) evaluated in fp64 and rounded
+ * to fp32, for x = 0..15 and x = 16 m.  One launch on `stream`. */
+cobra_status cobra_rope_table(double theta, int max_pos, float* table, size_t table_bytes, void* stream);
+
+/* RoPE decode attention with a planned workspace (cobra_decode_plan; the plan and the
+ * workspace are the same as for cobra_decode_attn).  q: device bf16; q_pos: device int32
+ * [n_seqs] query positions, or NULL for seq_lens[s] - 1; rope_table / max_pos: a table from
+ * cobra_rope_table.  A query position or sequence length outside the table, or a head whose
+ * code rows do not fit the kernel's staging, is reported through the device status word
+ * (cobra_check returns COBRA_EINVAL) and computed with clamped angles or skipped.  The
+ * reconstructed keys must stay below 2^14 Delta_K (|mu_K| small against Delta_K 2^15).
+ * Three launches: query rotation, scan, combine + back-projection; nothing is synchronised. */
+cobra_status cobra_decode_rope_attn(const void* params, const cobra_decode_desc* desc, const cobra_decode_info* info,
+                                    const void* q, const int* q_pos, const float* rope_table, int max_pos,
+                                    const uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
+                                    void* workspace, size_t ws_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------------
  * Decode attention without any device allocation.  (The paper has no counterpart; this is an
  * interface convenience.)
  *

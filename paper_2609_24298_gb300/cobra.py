@@ -97,6 +97,11 @@ SIGNATURES = {
                                      c_void_p, c_void_p, c_size_t, c_void_p]),
     "cobra_decode_attn_static": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), c_void_p, c_void_p, c_void_p, c_void_p,
                                          c_void_p, c_void_p]),
+    "cobra_rope_table_bytes": (c_int, [c_int, P_size]),
+    "cobra_rope_table": (c_int, [c_double, c_int, c_void_p, c_size_t, c_void_p]),
+    "cobra_decode_rope_attn": (c_int, [c_void_p, ctypes.POINTER(DecodeDesc), ctypes.POINTER(DecodeInfo), c_void_p,
+                                       c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p,
+                                       c_size_t, c_void_p]),
     "cobra_check": (c_int, [c_void_p]),
     "cobra_selftest_wait_timeout": (c_int, [ctypes.c_ulonglong, c_void_p]),
 }
@@ -403,6 +408,27 @@ def cobra_decode_combine(params, desc, info, seq_lens, out, workspace, ws_bytes:
     st = lib().cobra_decode_combine(_ptr(params), ctypes.byref(desc), ctypes.byref(info), _ptr(seq_lens), _ptr(out),
                                     _ptr(workspace), int(ws_bytes), _stream(stream))
     _chk("cobra_decode_combine", st)
+
+
+def cobra_rope_table_bytes(max_pos: int) -> int:
+    n = c_size_t(0)
+    _chk("cobra_rope_table_bytes", lib().cobra_rope_table_bytes(int(max_pos), ctypes.byref(n)))
+    return n.value
+
+
+def cobra_rope_table(theta: float, max_pos: int, table, table_bytes: int, stream=None):
+    """Fill a device angle table for RoPE decode (cos / sin of the rotary angles)."""
+    st = lib().cobra_rope_table(float(theta), int(max_pos), _ptr(table), int(table_bytes), _stream(stream))
+    _chk("cobra_rope_table", st)
+
+
+def cobra_decode_rope_attn(params, desc: DecodeDesc, info: DecodeInfo, q, q_pos, rope_table, max_pos: int, cache,
+                           seq_lens, page_table, out, workspace, ws_bytes: int, stream=None):
+    """Decode attention with the rotary embedding applied to the rebuilt keys and the query."""
+    st = lib().cobra_decode_rope_attn(_ptr(params), ctypes.byref(desc), ctypes.byref(info), _ptr(q), _ptr(q_pos),
+                                      _ptr(rope_table), int(max_pos), _ptr(cache), _ptr(seq_lens), _ptr(page_table),
+                                      _ptr(out), _ptr(workspace), int(ws_bytes), _stream(stream))
+    _chk("cobra_decode_rope_attn", st)
 
 
 def cobra_decode_attn_static(params, desc: DecodeDesc, q, cache, seq_lens, page_table, out, stream=None):

@@ -16,6 +16,7 @@
 #include "decode_heads.cuh"
 #include "measure.cuh"
 #include "calib.cuh"
+#include "rope.cuh"
 
 using namespace cobra;
 
@@ -300,10 +301,10 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
   return COBRA_OK;
 }
 
-cobra_status decode_common(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info, const void* q,
-                           const uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
-                           void* workspace, size_t ws_bytes, void* stream, int stages,
-                           const CompressArgs& ak = CompressArgs{}) {
+// Checks shared by the decode entry points and the kernel arguments they build.
+cobra_status decode_args(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info, const void* q,
+                         const uint8_t* cache, const int* seq_lens, const int* page_table, float* out, void* workspace,
+                         size_t ws_bytes, int stages, DecodeArgs& a) {
   if (!d || !info || !params || !workspace) return COBRA_EINVAL;
   if ((stages & kQproj) && !q) return COBRA_EINVAL;
   if ((stages & kScan) && (!cache || !seq_lens)) return COBRA_EINVAL;
@@ -316,7 +317,7 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   if (info->max_row_bytes < 0 || info->max_row_bytes > 16 * 128 * 8 || (info->max_row_bytes % 16)) return COBRA_EINVAL;
   if (ws_bytes < sizeof(WsHeader)) return COBRA_ESPACE;
   if (info->n_groups < 1 || info->n_items < 1) return COBRA_EINVAL;
-  DecodeArgs a{};
+  a = DecodeArgs{};
   a.block = static_cast<const unsigned char*>(params);
   a.cache = cache;
   a.seq_lens = seq_lens;
@@ -334,9 +335,21 @@ cobra_status decode_common(const void* params, const cobra_decode_desc* d, const
   const int rowb = info->max_row_bytes > 0 ? info->max_row_bytes : 16;
   // 8 KB of row staging per warp, or two of the largest rows if those are bigger
   a.ring_bytes = (int)std::max<size_t>(8192, 2 * align_up((size_t)rowb, 128));
-  cudaStream_t s = (cudaStream_t)stream;
   const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
   if (n_heads * d->n_seqs != info->n_groups) return COBRA_EINVAL;  // plan made for another descriptor
+  return COBRA_OK;
+}
+
+cobra_status decode_common(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info, const void* q,
+                           const uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
+                           void* workspace, size_t ws_bytes, void* stream, int stages,
+                           const CompressArgs& ak = CompressArgs{}) {
+  DecodeArgs a;
+  const cobra_status st =
+      decode_args(params, d, info, q, cache, seq_lens, page_table, out, workspace, ws_bytes, stages, a);
+  if (st != COBRA_OK) return st;
+  cudaStream_t s = (cudaStream_t)stream;
+  const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
   if (d->group == 4) return launch_decode<4>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak);
   return launch_decode<8>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak);
 }
@@ -412,6 +425,96 @@ extern "C" cobra_status cobra_decode_combine(const void* params, const cobra_dec
                                              void* workspace, size_t ws_bytes, void* stream) {
   return decode_common(params, d, info, nullptr, nullptr, seq_lens, nullptr, out, workspace, ws_bytes, stream,
                        kCombine);
+}
+
+// ---------------------------------------------------------------------------------------
+// Decode attention with the rotary position embedding applied after reconstruction.
+// ---------------------------------------------------------------------------------------
+namespace {
+
+constexpr int kRopeMaxPos = 1 << 22;
+
+int smem_optin() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  return n;
+}
+
+template <int G>
+cobra_status launch_rope(const DecodeArgs& a, const RopeArgs& ra0, int n_heads, int n_seqs, int n_items,
+                         int max_row_bytes, cudaStream_t s) {
+  RopeArgs ra = ra0;
+  // a stage holds the channel tiles of a K row (at most 2 KB past the row) and a V row; the
+  // two stages of a warp also hold its partial for the merge
+  const size_t rowb = (size_t)std::max(max_row_bytes, 16);
+  const size_t stage = std::max<size_t>(align_up(rowb + 2048, 128) + align_up(rowb, 128), 2560);
+  ra.stage_bytes = (int)stage;
+  const size_t fixed = rope_fixed_bytes<G>(), per_warp = rope_warp_bytes<G>((int)stage);
+  const long long room = (long long)smem_optin() - 1024 - (long long)fixed;
+  const int nw = (int)std::min<long long>(kRopeMaxWarps, room > 0 ? room / (long long)per_warp : 0);
+  if (nw < 1) return COBRA_EINVAL;  // code rows too large for the staging
+  const size_t smem = fixed + (size_t)nw * per_warp;
+  static size_t attr_set = 0;
+  if (smem > attr_set) {
+    if (cudaFuncSetAttribute(rope_scan_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess)
+      return COBRA_ECUDA;
+    attr_set = smem;
+  }
+  if (launch_pdl(rope_qprep_kernel<G>, (unsigned)n_heads, kHeadThreads, 0, s, a, ra) != cudaSuccess)
+    return COBRA_ECUDA;
+  // one CTA per SM; the work counter is 0 here (the plan writes it so, every scan resets it)
+  const int grid = std::max(1, std::min(n_items, sm_count()));
+  if (launch_pdl(rope_scan_kernel<G>, (unsigned)grid, nw * 32, smem, s, a, ra) != cudaSuccess) return COBRA_ECUDA;
+  return launch_decode<G>(a, n_heads, n_seqs, n_items, kCombine, s);
+}
+
+}  // namespace
+
+extern "C" cobra_status cobra_rope_table_bytes(int max_pos, size_t* bytes) {
+  if (!bytes || max_pos < 1 || max_pos > kRopeMaxPos) return COBRA_EINVAL;
+  *bytes = rope_table_floats((max_pos + kRopeFine - 1) / kRopeFine) * sizeof(float);
+  return COBRA_OK;
+}
+
+extern "C" cobra_status cobra_rope_table(double theta, int max_pos, float* table, size_t table_bytes, void* stream) {
+  size_t need = 0;
+  cobra_status st = cobra_rope_table_bytes(max_pos, &need);
+  if (st != COBRA_OK) return st;
+  if (!table || !(theta > 0.0) || !(theta < 1e300)) return COBRA_EINVAL;
+  if (!aligned(table, 16)) return COBRA_EALIGN;
+  if (table_bytes < need) return COBRA_ESPACE;
+  const int n_rows = kRopeFine + (max_pos + kRopeFine - 1) / kRopeFine;
+  const int n = n_rows * (kD / 2);
+  if (launch_pdl(rope_table_kernel, (unsigned)((n + 255) / 256), 256, 0, (cudaStream_t)stream, table, n_rows, theta) !=
+      cudaSuccess)
+    return COBRA_ECUDA;
+  return launch_status();
+}
+
+extern "C" cobra_status cobra_decode_rope_attn(const void* params, const cobra_decode_desc* d,
+                                               const cobra_decode_info* info, const void* q, const int* q_pos,
+                                               const float* rope_table, int max_pos, const uint8_t* cache,
+                                               const int* seq_lens, const int* page_table, float* out,
+                                               void* workspace, size_t ws_bytes, void* stream) {
+  if (!q || !cache || !seq_lens || !out || !rope_table) return COBRA_EINVAL;
+  if (max_pos < 1 || max_pos > kRopeMaxPos) return COBRA_EINVAL;
+  if (!aligned(rope_table, 16) || (q_pos && !aligned(q_pos, 4))) return COBRA_EALIGN;
+  DecodeArgs a;
+  const cobra_status st = decode_args(params, d, info, q, cache, seq_lens, page_table, out, workspace, ws_bytes,
+                                      kQproj | kScan | kCombine, a);
+  if (st != COBRA_OK) return st;
+  RopeArgs ra{};
+  ra.table = rope_table;
+  ra.q_pos = q_pos;
+  ra.n_coarse = (max_pos + kRopeFine - 1) / kRopeFine;
+  const int n_heads = d->n_layers * d->n_kv_heads;
+  cudaStream_t s = (cudaStream_t)stream;
+  cobra_status r = d->group == 4
+                       ? launch_rope<4>(a, ra, n_heads, d->n_seqs, info->n_items, info->max_row_bytes, s)
+                       : launch_rope<8>(a, ra, n_heads, d->n_seqs, info->n_items, info->max_row_bytes, s);
+  return r != COBRA_OK ? r : launch_status();
 }
 
 // ---------------------------------------------------------------------------------------

@@ -7,6 +7,7 @@ import torch
 
 from oracle import compress as ocomp
 from oracle import layout as olay
+from oracle import rope as orope
 from paper_2609_24298_gb300 import cobra, synth
 
 from .gpu_util import DEV, oracle_decode, oracle_head, oracle_heads_allocated, rel_err, upload
@@ -22,9 +23,10 @@ def need_gpu():
     cobra.lib()
 
 
-def run_decode(params, srcs, layers, kv, G, lens, q_scale=1.0, paged=False, seed=21, cap=None):
+def run_decode(params, srcs, layers, kv, G, lens, q_scale=1.0, paged=False, seed=21, cap=None, rope=None):
     """params/srcs in library order [K(l, h)..., V(l, h)...].  Packs the oracle's codes into the
-    cache, runs the library's decode, returns (out, reference)."""
+    cache, runs the library's decode, returns (out, reference).  rope = dict(theta, q_pos
+    (per sequence, or None for len - 1), max_pos) runs the RoPE decode against oracle.rope."""
     seqs = len(lens)
     cap = np.asarray(cap if cap is not None else lens, np.int32)
     rows_per_seq = max(1, int(-(-cap.max() // 128)))
@@ -69,7 +71,16 @@ def run_decode(params, srcs, layers, kv, G, lens, q_scale=1.0, paged=False, seed
     out = torch.full((layers, seqs, kv * G, 128), float("nan"), dtype=torch.float32, device=DEV)
     lens_d = torch.tensor(np.asarray(lens, np.int32), device=DEV)
     pt = torch.tensor(page_table.reshape(-1), dtype=torch.int32, device=DEV) if paged else None
-    cobra.cobra_decode_attn(block, desc, info, qd, cache, lens_d, pt, out, ws, wsb)
+    if rope is None:
+        cobra.cobra_decode_attn(block, desc, info, qd, cache, lens_d, pt, out, ws, wsb)
+    else:
+        max_pos = rope.get("max_pos") or max(1, int(cap.max()))
+        tb = cobra.cobra_rope_table_bytes(max_pos)
+        table = torch.empty(tb // 4, dtype=torch.float32, device=DEV)
+        cobra.cobra_rope_table(rope["theta"], max_pos, table, tb)
+        qp = rope.get("q_pos")
+        qpd = torch.tensor(np.asarray(qp, np.int32), device=DEV) if qp is not None else None
+        cobra.cobra_decode_rope_attn(block, desc, info, qd, qpd, table, max_pos, cache, lens_d, pt, out, ws, wsb)
     assert cobra.cobra_check() == cobra.COBRA_OK
     o = out.cpu().numpy()
     ref = np.zeros_like(o, dtype=np.float64)
@@ -78,7 +89,14 @@ def run_decode(params, srcs, layers, kv, G, lens, q_scale=1.0, paged=False, seed
             ik, iv = l * kv + h, n + l * kv + h
             for q in range(seqs):
                 qq = qh[l, q, h * G:(h + 1) * G].astype(np.float64)
-                ref[l, q, h * G:(h + 1) * G] = oracle_decode(qq, codes[(ik, q)], codes[(iv, q)], params[ik], params[iv])
+                if rope is None:
+                    ref[l, q, h * G:(h + 1) * G] = oracle_decode(qq, codes[(ik, q)], codes[(iv, q)], params[ik],
+                                                                 params[iv])
+                elif lens[q] > 0:
+                    qp = rope.get("q_pos")
+                    pos = int(qp[q]) if qp is not None else int(lens[q]) - 1
+                    ref[l, q, h * G:(h + 1) * G] = orope.decode(qq, codes[(ik, q)], codes[(iv, q)], params[ik],
+                                                                params[iv], pos, rope["theta"])
     return o, ref, info
 
 

@@ -206,3 +206,35 @@ def test_selftest_wait_limits_checked_before_launch():
     for bad in (0, 100_000_001):
         with pytest.raises(Exception):
             cobra.cobra_selftest_wait_timeout(bad)
+
+
+def test_rope_entry_points_check_arguments_before_the_gpu(L):
+    # table: 16 fine rows + one row per 16 positions, 128 floats each
+    assert cobra.cobra_rope_table_bytes(1) == 17 * 128 * 4
+    assert cobra.cobra_rope_table_bytes(32768) == (16 + 2048) * 128 * 4
+    assert cobra.cobra_rope_table_bytes(33) == (16 + 3) * 128 * 4
+    for bad in (0, (1 << 22) + 1):
+        with pytest.raises(cobra.CobraError) as e:
+            cobra.cobra_rope_table_bytes(bad)
+        assert e.value.status == cobra.COBRA_EINVAL
+    need = cobra.cobra_rope_table_bytes(100)
+    for theta, table, nbytes, status in ((0.0, 256, need, cobra.COBRA_EINVAL), (float("nan"), 256, need, cobra.COBRA_EINVAL),
+                                         (1e4, None, need, cobra.COBRA_EINVAL), (1e4, 264, need, cobra.COBRA_EALIGN),
+                                         (1e4, 256, need - 16, cobra.COBRA_ESPACE)):
+        with pytest.raises(cobra.CobraError) as e:
+            cobra.cobra_rope_table(theta, 100, table, nbytes)
+        assert e.value.status == status
+    d4 = cobra.decode_desc(k_head0=0, v_head0=1, layer_stride=1, n_layers=1, n_kv_heads=1, group=4, n_seqs=1,
+                           rows_per_seq=1)
+    d3 = cobra.decode_desc(k_head0=0, v_head0=1, layer_stride=1, n_layers=1, n_kv_heads=1, group=3, n_seqs=1,
+                           rows_per_seq=1)
+    info = cobra.DecodeInfo(1, 1, 16, 0)
+    cases = [(d4, None, 256, 256, 10, cobra.COBRA_EINVAL),  # no query
+             (d4, 256, 256, 264, 10, cobra.COBRA_EALIGN),   # table not 16-byte aligned
+             (d4, 256, 258, 256, 10, cobra.COBRA_EALIGN),   # q_pos not 4-byte aligned
+             (d4, 256, 256, 256, 0, cobra.COBRA_EINVAL),    # no positions
+             (d3, 256, 256, 256, 10, cobra.COBRA_EINVAL)]   # group of 3
+    for desc, q, qpos, table, max_pos, status in cases:
+        with pytest.raises(cobra.CobraError) as e:
+            cobra.cobra_decode_rope_attn(256, desc, info, q, qpos, table, max_pos, 256, 256, None, 256, 256, 1 << 20)
+        assert e.value.status == status
