@@ -58,6 +58,8 @@ def parse_args():
     ap.add_argument("--measured-only", action="store_true", help="only the measured distortion tables")
     ap.add_argument("--no-calibration", action="store_true", help="skip the device calibration leg")
     ap.add_argument("--calibration-only", action="store_true", help="only the device calibration leg")
+    ap.add_argument("--no-rope", action="store_true", help="skip the RoPE decode leg")
+    ap.add_argument("--rope-steps", type=int, default=20, help="timed calls of the RoPE decode leg")
     return ap.parse_args()
 
 
@@ -203,6 +205,24 @@ class OracleSample:
             _, c = ocomp.compress(self.new[side], p["W"], p["mu"], p["delta"], SAMPLE_B)
             codes.append(np.concatenate([self.codes[side], c]))
         return oatt.decode(self.q, codes[0], codes[1], self.params[0], self.params[1])
+
+
+def oracle_rope_rate(seconds: float, T: int, group: int):
+    """Packed bytes per second the oracle's RoPE decode (oracle/rope.py) processes over the
+    context of OracleSample groups, timed over about `seconds` of work."""
+    from oracle import rope as orope
+
+    samples = [OracleSample(h, T, group) for h in range(2)]
+    done, nbytes, t0 = 0, 0, time.perf_counter()
+    while True:
+        s = samples[done % len(samples)]
+        orope.decode(s.q, s.codes[0], s.codes[1], s.params[0], s.params[1], T - 2, ROPE_THETA)
+        nbytes += s.bytes
+        done += 1
+        el = time.perf_counter() - t0
+        if el >= seconds and done >= 2:
+            break
+    return nbytes / el / 1e9, done, el
 
 
 def oracle_rate(seconds: float, T: int, group: int):
@@ -517,6 +537,83 @@ def run_measured_leg(args, dev, stream, cals, srcs, cpu_baseline: bool):
 # ---------------------------------------------------------------------------------------
 # the CUDA path
 # ---------------------------------------------------------------------------------------
+ROPE_THETA = 500000.0  # Llama-3-8B's rotary base
+ROPE_SOURCES = ["paper_2609_24298_gb300/csrc/rope.cuh", "paper_2609_24298_gb300/csrc/decode.cuh",
+                "paper_2609_24298_gb300/csrc/common.cuh"]
+ROPE_PROFILE = os.path.join(ROOT, "profiles", "rope_decode_llama3_8b.txt")
+
+
+def bf16_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 1900.0, "fallback"
+
+
+def run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out, cpu_baseline: bool):
+    """Decode attention for a model with the rotary embedding (K compressed before it, Sec. 5
+    "Scope"): the same compressed cache, plan and queries as the main step, each key rebuilt,
+    turned to its position and scored (cobra_decode_rope_attn, three launches).  The rebuild is
+    a dense contraction, so the leg is measured against the tensor roofline: algorithmic
+    FLOPs per call = sum over (seq, layer, kv head) of T (2 d r_K + 2 d G + 2 r_V G).
+    Returns the JSON object reported under "rope"."""
+    import torch
+
+    from paper_2609_24298_gb300 import cobra, pipeline
+
+    L, H, S, G = wl.layers, wl.kv, wl.seqs, wl.group
+    T = int(np.max(wl.tokens))
+    cpu = None
+    if cpu_baseline:
+        gbs, n, el = oracle_rope_rate(min(args.cpu_seconds, 10.0), T, G)
+        cpu = {"value": gbs, "unit": "GB/s", "cores": cores_used(), "kind": "oracle",
+               "sample": f"{n} (seq, layer, kv-head) RoPE decodes over {T - 1} tokens with K and V at "
+                         f"r={SAMPLE_R}, b={SAMPLE_B} ({el:.1f} s of fp64 numpy)"}
+    tb = cobra.cobra_rope_table_bytes(T)
+    table = torch.empty(tb // 4, dtype=torch.float32, device=dev)
+    cobra.cobra_rope_table(ROPE_THETA, T, table, tb, stream)
+    nws = ws.numel()
+
+    def call():
+        cobra.cobra_decode_rope_attn(wl.dev.block, desc, info, q, None, table, T, wl.dev.cache, lens, None, out, ws,
+                                     nws, stream)
+
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    if cobra.cobra_check(stream) != cobra.COBRA_OK:
+        raise RuntimeError("device status after the RoPE warm-up")
+    K = max(3, args.rope_steps)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(K):
+        call()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if cobra.cobra_check(stream) != cobra.COBRA_OK:
+        raise RuntimeError("device status after the RoPE timed region")
+    ms = e0.elapsed_time(e1) / K
+    n = L * H
+    rk = np.asarray(hp.r[:n], np.float64)
+    rv = np.asarray(hp.r[n:2 * n], np.float64)
+    flops = float(S * T * np.sum(2 * 128 * rk + 2 * 128 * G + 2 * rv * G))
+    bytes_call = pipeline.packed_bytes_read(wl)
+    peak, kind = bf16_peak()
+    achieved = flops / (ms * 1e-3) / 1e12
+    return {"metric": "packed KV bytes decoded per second with RoPE", "value": bytes_call / (ms * 1e-3) / 1e9,
+            "unit": "GB/s", "ms_per_call": ms, "calls": K, "theta": ROPE_THETA,
+            "workload": f"the main step's cache and queries: {L} layers x {H} kv heads x {S} seqs x {T} tokens, "
+                        "query at position T - 1",
+            "roofline": {"bound": "tensor", "kernel": "rope_scan_kernel (timed with its query rotation and "
+                                                      "combine launches)",
+                         "achieved": achieved, "peak": peak, "peak_kind": kind + " bf16 burst", "unit": "TFLOP/s",
+                         "frac": achieved / peak, "algorithmic_flops_per_call": flops,
+                         "traffic": profiled_value("traffic_bytes_per_launch", ROPE_PROFILE, ROPE_SOURCES)},
+            "cpu_baseline": cpu,
+            "gpu_launches": 3 * K}
+
+
 def run_cobra(args):
     import torch
     import torch.distributed as dist
@@ -707,6 +804,10 @@ def run_cobra(args):
     measured = None
     if not args.no_measured and rank == 0:
         measured = run_measured_leg(args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
+    rope = None
+    if not args.no_rope and rank == 0:
+        rope = run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out,
+                            not args.no_cpu_baseline and world == 1)
     compress = None
     if not args.no_compress:
         del hin, hout
@@ -724,6 +825,7 @@ def run_cobra(args):
                          "traffic": traffic, "scan_ms": scan_ms,
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
             "compress": compress,
+            "rope": rope,
             "measured": measured,
             "calibration": calibration,
             "cpu_baseline": cpu,

@@ -263,7 +263,8 @@ typedef struct {
   int n_groups;       /* (seq, layer, kv-head) triples */
   int n_items;        /* token chunks */
   int max_row_bytes;  /* largest K or V code row among the planned heads */
-  int reserved;
+  int max_stage_bytes; /* largest K row in whole 16-channel tiles plus V row (128-byte aligned)
+                          of a group, for the RoPE decode's staging (0: not known) */
 } cobra_decode_info;
 
 /* Write the work plan (token chunks of whole code rows per (seq, layer, kv-head), in the order

@@ -47,7 +47,7 @@ class DecodeDesc(ctypes.Structure):
 
 
 class DecodeInfo(ctypes.Structure):
-    _fields_ = [("n_groups", c_int), ("n_items", c_int), ("max_row_bytes", c_int), ("reserved", c_int)]
+    _fields_ = [("n_groups", c_int), ("n_items", c_int), ("max_row_bytes", c_int), ("max_stage_bytes", c_int)]
 
 
 # name -> (restype, argtypes)

@@ -750,6 +750,7 @@ struct Plan {
   std::vector<cobra::WsGroup> groups;
   std::vector<cobra::WsItem> items;
   int max_rv = 0, max_row_bytes = 0;
+  int max_stage_bytes = 0;  // largest K channel tiles + V row (128-byte aligned) of a group
 };
 
 cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int* head_b, const int* seq_cap, Plan& p) {
@@ -792,6 +793,8 @@ cobra_status make_plan(const cobra_decode_desc* d, const int* head_r, const int*
     p.max_rv = std::max(p.max_rv, key.rv);
     p.max_row_bytes =
         std::max(p.max_row_bytes, (int)std::max(cobra_row_bytes(key.rk, key.bk), cobra_row_bytes(key.rv, key.bv)));
+    p.max_stage_bytes = std::max(p.max_stage_bytes, 256 * key.bk * ((key.rk + 15) / 16) +
+                                                        (int)align_up(cobra_row_bytes(key.rv, key.bv), 128));
     const long long rows = (seq_cap[key.s] + 127) / 128, rb = pair_bytes(key);
     cobra::WsGroup g{key.s, key.l, key.h, (int)p.items.size(), 0, hk, hv, 0};
     if (rows == 0 || rb == 0) {  // one (empty or code-less) chunk
@@ -876,7 +879,7 @@ cobra_status plan_image(const cobra_decode_desc* desc, const int* head_r, const 
   info->n_groups = h.n_groups;
   info->n_items = h.n_items;
   info->max_row_bytes = h.max_row_bytes;
-  info->reserved = 0;
+  info->max_stage_bytes = p.max_stage_bytes;
   return COBRA_OK;
 }
 }  // namespace

@@ -315,6 +315,7 @@ cobra_status decode_args(const void* params, const cobra_decode_desc* d, const c
       (q && !aligned(q, 2)))
     return COBRA_EALIGN;
   if (info->max_row_bytes < 0 || info->max_row_bytes > 16 * 128 * 8 || (info->max_row_bytes % 16)) return COBRA_EINVAL;
+  if (info->max_stage_bytes < 0 || info->max_stage_bytes > 2 * 16 * 128 * 8) return COBRA_EINVAL;
   if (ws_bytes < sizeof(WsHeader)) return COBRA_ESPACE;
   if (info->n_groups < 1 || info->n_items < 1) return COBRA_EINVAL;
   a = DecodeArgs{};
@@ -442,13 +443,16 @@ int smem_optin() {
 }
 
 template <int G>
-cobra_status launch_rope(const DecodeArgs& a, const RopeArgs& ra0, int n_heads, int n_seqs, int n_items,
-                         int max_row_bytes, cudaStream_t s) {
+cobra_status launch_rope(const DecodeArgs& a, const RopeArgs& ra0, int n_heads, int n_seqs, int n_groups,
+                         int n_items, int max_row_bytes, int max_stage_bytes, cudaStream_t s) {
   RopeArgs ra = ra0;
-  // a stage holds the channel tiles of a K row (at most 2 KB past the row) and a V row; the
-  // two stages of a warp also hold its partial for the merge
+  // a stage holds the channel tiles of a K row and a V row: the plan's largest, else a bound
+  // from the largest row (at most 1792 bytes of tiles past a K row); the two stages of a warp
+  // also hold its partial for the merge
   const size_t rowb = (size_t)std::max(max_row_bytes, 16);
-  const size_t stage = std::max<size_t>(align_up(rowb + 2048, 128) + align_up(rowb, 128), 2560);
+  const size_t need = max_stage_bytes > 0 ? (size_t)max_stage_bytes
+                                          : align_up(rowb + 1792, 128) + align_up(rowb, 128);
+  const size_t stage = std::max<size_t>(align_up(need, 128), 2560);
   ra.stage_bytes = (int)stage;
   const size_t fixed = rope_fixed_bytes<G>(), per_warp = rope_warp_bytes<G>((int)stage);
   const long long room = (long long)smem_optin() - 1024 - (long long)fixed;
@@ -464,8 +468,9 @@ cobra_status launch_rope(const DecodeArgs& a, const RopeArgs& ra0, int n_heads, 
   }
   if (launch_pdl(rope_qprep_kernel<G>, (unsigned)n_heads, kHeadThreads, 0, s, a, ra) != cudaSuccess)
     return COBRA_ECUDA;
-  // one CTA per SM; the work counter is 0 here (the plan writes it so, every scan resets it)
-  const int grid = std::max(1, std::min(n_items, sm_count()));
+  // one CTA per SM over the groups; the work counter is 0 here (the plan writes it so, every
+  // scan resets it)
+  const int grid = std::max(1, std::min(n_groups, sm_count()));
   if (launch_pdl(rope_scan_kernel<G>, (unsigned)grid, nw * 32, smem, s, a, ra) != cudaSuccess) return COBRA_ECUDA;
   return launch_decode<G>(a, n_heads, n_seqs, n_items, kCombine, s);
 }
@@ -512,8 +517,10 @@ extern "C" cobra_status cobra_decode_rope_attn(const void* params, const cobra_d
   const int n_heads = d->n_layers * d->n_kv_heads;
   cudaStream_t s = (cudaStream_t)stream;
   cobra_status r = d->group == 4
-                       ? launch_rope<4>(a, ra, n_heads, d->n_seqs, info->n_items, info->max_row_bytes, s)
-                       : launch_rope<8>(a, ra, n_heads, d->n_seqs, info->n_items, info->max_row_bytes, s);
+                       ? launch_rope<4>(a, ra, n_heads, d->n_seqs, info->n_groups, info->n_items,
+                                        info->max_row_bytes, info->max_stage_bytes, s)
+                       : launch_rope<8>(a, ra, n_heads, d->n_seqs, info->n_groups, info->n_items,
+                                        info->max_row_bytes, info->max_stage_bytes, s);
   return r != COBRA_OK ? r : launch_status();
 }
 

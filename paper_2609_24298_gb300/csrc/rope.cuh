@@ -20,13 +20,14 @@
 //   rope_qprep_kernel  q' = (Delta_K / sqrt d) log2(e) R(p) q per query head, scaled by a
 //                      power of two, split into fp16 hi + lo and laid out as the score MMA's
 //                      B fragments in the workspace's q~ block of the group.
-//   rope_scan_kernel   CTAs take the decode plan's work items; the CTA's warps share the
-//                      item's rows.  Per pair of 16-token tiles and 16 channel positions:
+//   rope_scan_kernel   CTAs take whole (seq, layer, kv head) groups of the decode plan; the
+//                      CTA's warps share the group's rows.  Per pair of 16-token tiles:
 //                        rebuild  X = seed + A W'   (A the unpacked codes, W' = W_K^T hi + lo)
 //                        turn     X <- R(t) X       (the token's composed angle, per pair)
 //                        score    S += X q'         (X and q' both split hi + lo)
 //                      followed by the scan's online softmax and rank-space accumulation of
-//                      V (not rotated), and a merge of the CTA's warps into the item's partial.
+//                      V (not rotated), and a merge of the CTA's warps into the first of the
+//                      group's partial slots (the others are left empty for combine_kernel).
 //   combine_kernel     (decode_heads.cuh) as for the plain decode.
 //
 // The codes unpack to A = 1 + c 2^(k - 10) with the per-register window k of the scan (see
@@ -46,6 +47,7 @@ constexpr int kRopeMaxWarps = 8;
 constexpr int kRopeKTiles = 8;        // channel tiles of 16 (r <= 128)
 constexpr int kRopeSeedSlots = 8;     // windows k = 2 .. 9
 constexpr int kRopeMergeStride = 4 + kD;  // floats per query head in a warp's partial
+constexpr int kRopeCh = 2;            // blocks of 16 positions rebuilt per pass over the codes
 
 // Table entry of pair j = 4 n + jj within a row: [(jj * 16 + n) * 2 + (0: cos, 1: sin)].  The
 // two pairs (8 ch + jj, 8 ch + 4 + jj) that a lane turns in channel block ch are one float4.
@@ -204,7 +206,7 @@ __global__ void __launch_bounds__(kHeadThreads) rope_qprep_kernel(DecodeArgs a, 
 // B = 0 stands for a head without K codes (r_K = 0).
 //   wfrag  W' B fragments [kt][n-tile][hi, lo][lane] (channels past r are zero)
 //   seed4  [slot][ch][jj] float4: positions 16 ch + 2 jj + {0, 1, 8, 9} of window slot k - 2
-//   fine4  fine table rows as float4; coarse4 the coarse rows (global)
+//   fine4  fine table entries as float4 [jj][ch][i]; coarse4 the coarse rows (global)
 //   crow   coarse row of the row's first token tile (token 128 row -> 8 row)
 // ---------------------------------------------------------------------------------------
 template <int B>
@@ -238,81 +240,99 @@ __device__ __forceinline__ void rope_k_row(const uint8_t* stage, int rk, int cro
 #pragma unroll
     for (int mi = 0; mi < 2; ++mi) co[mi] = coarse4 + (size_t)min(crow + 2 * mp + mi, n_coarse - 1) * (kRopeRowFloats / 4);
 #pragma unroll 1
-    for (int ch = 0; ch < 8; ++ch) {
-      // rebuild X for n-tiles 2 ch, 2 ch + 1 of both token tiles, starting from the seeds
-      float x[2][2][4];
+    for (int ch0 = 0; ch0 < 8; ch0 += kRopeCh) {
+      // rebuild X for n-tiles 2 ch, 2 ch + 1 (ch = ch0 .. ch0 + kRopeCh - 1) of both token
+      // tiles, starting from the seeds
+      float x[2][kRopeCh][2][4];
 #pragma unroll
       for (int mi = 0; mi < 2; ++mi) {
         const int t = 2 * mp + mi;
-        const float4 sl = seed4[(rope_slot<B>(2 * t) * 8 + ch) * 4 + jj];
-        const float4 sh = seed4[(rope_slot<B>(2 * t + 1) * 8 + ch) * 4 + jj];
-        x[mi][0][0] = sl.x;
-        x[mi][0][1] = sl.y;
-        x[mi][0][2] = sh.x;
-        x[mi][0][3] = sh.y;
-        x[mi][1][0] = sl.z;
-        x[mi][1][1] = sl.w;
-        x[mi][1][2] = sh.z;
-        x[mi][1][3] = sh.w;
+#pragma unroll
+        for (int c = 0; c < kRopeCh; ++c) {
+          const float4 sl = seed4[(rope_slot<B>(2 * t) * 8 + ch0 + c) * 4 + jj];
+          const float4 sh = seed4[(rope_slot<B>(2 * t + 1) * 8 + ch0 + c) * 4 + jj];
+          x[mi][c][0][0] = sl.x;
+          x[mi][c][0][1] = sl.y;
+          x[mi][c][0][2] = sh.x;
+          x[mi][c][0][3] = sh.y;
+          x[mi][c][1][0] = sl.z;
+          x[mi][c][1][1] = sl.w;
+          x[mi][c][1][2] = sh.z;
+          x[mi][c][1][3] = sh.w;
+        }
       }
       if constexpr (B > 0) {
-        // the codes of both token tiles are unpacked again for every block of 16 positions:
-        // holding them for all channel tiles would not fit the registers
+        // the codes of both token tiles are unpacked again for every kRopeCh blocks of 16
+        // positions: holding them for all channel tiles would not fit the registers
 #pragma unroll 1
         for (int kt = 0; kt < nk; ++kt) {
           uint32_t wa[B], wb[B];
           load_piece<B>(pa + kt * 8 * 32 * B, wa);
           load_piece<B>(pa + kt * 8 * 32 * B + 4 * 32 * B, wb);
-          const uint2* wf = wfrag + (size_t)((kt * 16 + 2 * ch) * 2) * 32 + lane;
-          const uint2 b00 = wf[0], b01 = wf[32], b10 = wf[64], b11 = wf[96];  // [n-tile][hi, lo]
+          uint32_t av[2][4];
 #pragma unroll
           for (int mi = 0; mi < 2; ++mi) {
             const int t = 2 * mp + mi;
-            const uint32_t a0 = unpack_reg<B>(wa, 2 * t, one), a1 = unpack_reg<B>(wa, 2 * t + 1, one);
-            const uint32_t a2 = unpack_reg<B>(wb, 2 * t, one), a3 = unpack_reg<B>(wb, 2 * t + 1, one);
-            mma_f16(x[mi][0], a0, a1, a2, a3, b00.x, b00.y);
-            mma_f16(x[mi][0], a0, a1, a2, a3, b01.x, b01.y);
-            mma_f16(x[mi][1], a0, a1, a2, a3, b10.x, b10.y);
-            mma_f16(x[mi][1], a0, a1, a2, a3, b11.x, b11.y);
+            av[mi][0] = unpack_reg<B>(wa, 2 * t, one);
+            av[mi][1] = unpack_reg<B>(wa, 2 * t + 1, one);
+            av[mi][2] = unpack_reg<B>(wb, 2 * t, one);
+            av[mi][3] = unpack_reg<B>(wb, 2 * t + 1, one);
+          }
+#pragma unroll
+          for (int c = 0; c < kRopeCh; ++c) {
+            const uint2* wf = wfrag + (size_t)((kt * 16 + 2 * (ch0 + c)) * 2) * 32 + lane;
+            const uint2 bw[2][2] = {{wf[0], wf[32]}, {wf[64], wf[96]}};  // [n-tile][hi, lo]
+            // the hi and lo products of an accumulator are issued four MMAs apart
+#pragma unroll
+            for (int limb = 0; limb < 2; ++limb)
+#pragma unroll
+              for (int mi = 0; mi < 2; ++mi)
+#pragma unroll
+                for (int nn = 0; nn < 2; ++nn)
+                  mma_f16(x[mi][c][nn], av[mi][0], av[mi][1], av[mi][2], av[mi][3], bw[nn][limb].x, bw[nn][limb].y);
           }
         }
       }
-      // turn each pair (x[..][2h], x[..][2h+1]) by its token's angle: pair 8 ch + jj in
-      // n-tile 2 ch, 8 ch + 4 + jj in n-tile 2 ch + 1; token row gi (h = 0) or gi + 8 (h = 1)
-      const float4 f0 = fine4[gi * 32 + jj * 8 + ch], f1 = fine4[(gi + 8) * 32 + jj * 8 + ch];
 #pragma unroll
-      for (int mi = 0; mi < 2; ++mi) {
-        const float4 cm = __ldg(co[mi] + jj * 8 + ch);
+      for (int c = 0; c < kRopeCh; ++c) {
+        const int ch = ch0 + c;
+        // turn each pair (x[..][2h], x[..][2h+1]) by its token's angle: pair 8 ch + jj in
+        // n-tile 2 ch, 8 ch + 4 + jj in n-tile 2 ch + 1; token row gi (h = 0) or gi + 8 (h = 1)
+        const float4 f0 = fine4[(jj * 8 + ch) * kRopeFine + gi], f1 = fine4[(jj * 8 + ch) * kRopeFine + gi + 8];
 #pragma unroll
-        for (int nn = 0; nn < 2; ++nn) {
-          const float c0 = nn ? cm.z : cm.x, s0 = nn ? cm.w : cm.y;
+        for (int mi = 0; mi < 2; ++mi) {
+          const float4 cm = __ldg(co[mi] + jj * 8 + ch);
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const float4 f = h ? f1 : f0;
-            float c, sn;
-            rope_compose(c0, s0, nn ? f.z : f.x, nn ? f.w : f.y, c, sn);
-            const float xa = x[mi][nn][2 * h], xb = x[mi][nn][2 * h + 1];
-            x[mi][nn][2 * h] = fmaf(xa, c, -xb * sn);
-            x[mi][nn][2 * h + 1] = fmaf(xa, sn, xb * c);
+          for (int nn = 0; nn < 2; ++nn) {
+            const float c0 = nn ? cm.z : cm.x, s0 = nn ? cm.w : cm.y;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const float4 f = h ? f1 : f0;
+              float cs, sn;
+              rope_compose(c0, s0, nn ? f.z : f.x, nn ? f.w : f.y, cs, sn);
+              const float xa = x[mi][c][nn][2 * h], xb = x[mi][c][nn][2 * h + 1];
+              x[mi][c][nn][2 * h] = fmaf(xa, cs, -xb * sn);
+              x[mi][c][nn][2 * h + 1] = fmaf(xa, sn, xb * cs);
+            }
           }
         }
-      }
-      // the two n-tiles' accumulators are the A fragment of the k-tile of positions
-      // 16 ch .. 16 ch + 15 for the score MMA against q' (hi and lo of both sides)
-      uint2 bq[NTK];
+        // the two n-tiles' accumulators are the A fragment of the k-tile of positions
+        // 16 ch .. 16 ch + 15 for the score MMA against q' (hi and lo of both sides)
+        uint2 bq[NTK];
 #pragma unroll
-      for (int nt = 0; nt < NTK; ++nt) bq[nt] = qfrag[(ch * NTK + nt) * 32 + lane];
+        for (int nt = 0; nt < NTK; ++nt) bq[nt] = qfrag[(ch * NTK + nt) * 32 + lane];
 #pragma unroll
-      for (int mi = 0; mi < 2; ++mi) {
-        uint32_t h[4], l[4];
-        split_f16x2(x[mi][0][0], x[mi][0][1], h[0], l[0]);
-        split_f16x2(x[mi][0][2], x[mi][0][3], h[1], l[1]);
-        split_f16x2(x[mi][1][0], x[mi][1][1], h[2], l[2]);
-        split_f16x2(x[mi][1][2], x[mi][1][3], h[3], l[3]);
+        for (int mi = 0; mi < 2; ++mi) {
+          uint32_t h[4], l[4];
+          split_f16x2(x[mi][c][0][0], x[mi][c][0][1], h[0], l[0]);
+          split_f16x2(x[mi][c][0][2], x[mi][c][0][3], h[1], l[1]);
+          split_f16x2(x[mi][c][1][0], x[mi][c][1][1], h[2], l[2]);
+          split_f16x2(x[mi][c][1][2], x[mi][c][1][3], h[3], l[3]);
 #pragma unroll
-        for (int nt = 0; nt < NTK; ++nt) {
-          mma_f16(sacc[mi][nt], h[0], h[1], h[2], h[3], bq[nt].x, bq[nt].y);
-          mma_f16(sacc[mi][nt], l[0], l[1], l[2], l[3], bq[nt].x, bq[nt].y);
+          for (int nt = 0; nt < NTK; ++nt) {
+            mma_f16(sacc[mi][nt], h[0], h[1], h[2], h[3], bq[nt].x, bq[nt].y);
+            mma_f16(sacc[mi][nt], l[0], l[1], l[2], l[3], bq[nt].x, bq[nt].y);
+          }
         }
       }
     }
@@ -359,9 +379,10 @@ __device__ __forceinline__ void warp_copy_async(uint8_t* dst, const uint8_t* src
 }
 
 // ---------------------------------------------------------------------------------------
-// The scan: one CTA per SM takes work items from the plan's counter; its warps take the
-// item's rows in turn, each with its own softmax state and V accumulators, and the warps'
-// partials are merged into the item's slot.
+// The scan: one CTA per SM takes (seq, layer, kv head) groups from the plan's counter (W_K is
+// staged once per group, and whole groups keep the warps' shares of rows even); its warps take
+// the group's rows in turn, each with its own softmax state and V accumulators, and the warps'
+// partials are merged into the group's first slot.
 // ---------------------------------------------------------------------------------------
 template <int G>
 __global__ void __launch_bounds__(kRopeMaxWarps * 32, 1) rope_scan_kernel(DecodeArgs a, RopeArgs ra) {
@@ -382,25 +403,27 @@ __global__ void __launch_bounds__(kRopeMaxWarps * 32, 1) rope_scan_kernel(Decode
 
   const WsHeader* wh = reinterpret_cast<const WsHeader*>(a.ws);
   const WsGroup* groups = reinterpret_cast<const WsGroup*>(a.ws + wh->groups_off);
-  const WsItem* items = reinterpret_cast<const WsItem*>(a.ws + wh->items_off);
   const HeadEntry* heads = head_table(a.block);
   const float* pool = param_pool(a.block);
   float* parts = reinterpret_cast<float*>(a.ws + wh->part_off);
-  const int n_items = wh->n_items, gstride = wh->g_stride, pstride = wh->part_stride;
+  const int n_groups = wh->n_groups, gstride = wh->g_stride, pstride = wh->part_stride;
   unsigned int* next_item = const_cast<unsigned int*>(&wh->next_item);
   const float4* coarse4 = reinterpret_cast<const float4*>(ra.table + (size_t)kRopeFine * kRopeRowFloats);
-  for (int i = tid; i < (int)(kRopeFineBytes / 16); i += blockDim.x)
-    fine4[i] = reinterpret_cast<const float4*>(ra.table)[i];
+  // fine rows in shared memory as [jj][ch][i] float4, so that the lanes of a warp (token i =
+  // lane / 4 or + 8, pair group jj = lane % 4) read distinct banks
+  for (int idx = tid; idx < (int)(kRopeFineBytes / 16); idx += blockDim.x) {
+    const int i = idx / 32, q = idx % 32;  // table float4 q = jj * 8 + ch of fine row i
+    fine4[q * kRopeFine + i] = reinterpret_cast<const float4*>(ra.table)[idx];
+  }
   const uint32_t one = a.one;
   int staged_head = -1;
 
   for (;;) {
     if (tid == 0) s_item = (int)atomicAdd(next_item, 1u);
-    __syncthreads();  // (also: every warp is done with the previous item's shared memory)
-    const int item = s_item;
-    if (item >= n_items) break;
-    const WsItem it = items[item];
-    const WsGroup gr = groups[it.group];
+    __syncthreads();  // (also: every warp is done with the previous group's shared memory)
+    const int grp = s_item;
+    if (grp >= n_groups) break;
+    const WsGroup gr = groups[grp];
     const HeadEntry hk = heads[gr.k_head], hv = heads[gr.v_head];
     const int rk = hk.r, kb = hk.b, vr = hv.r, vb = hv.b;
     const int nk = (rk + 15) >> 4;
@@ -423,30 +446,34 @@ __global__ void __launch_bounds__(kRopeMaxWarps * 32, 1) rope_scan_kernel(Decode
         wfrag[idx] = make_uint2(pack_f16(v[0], v[1]), pack_f16(v[2], v[3]));
       }
       // seeds of every window slot: 2^(k-10) (mu'/Delta - c_b W'1) - W'1, or mu' when r = 0
+      // (one warp per position: the lanes sum W'1 over the channels, lane k - 2 writes slot k)
       float* seed = reinterpret_cast<float*>(seed4);
-      for (int P = tid; P < kD; P += blockDim.x) {
+      for (int P = warp; P < kD; P += nw) {
         const int dm = (P >> 1) + (P & 1) * (kD / 2);
         float w1 = 0.f;
-        for (int c = 0; c < rk; ++c) w1 += W[(size_t)c * kD + dm];
-        const float mu = pool[hk.mu_off + dm];
-        const float base = rk > 0 ? mu / hk.delta - ((float)(1 << (kb - 1)) - 0.5f) * w1 : 0.f;
-        const int ch = P >> 4, hi8 = (P >> 3) & 1, jq = (P >> 1) & 3, e = P & 1;
-        for (int slot = 0; slot < kRopeSeedSlots; ++slot) {
-          const float v = rk > 0 ? ldexpf(base, slot + 2 - 10) - w1 : (slot == 0 ? mu : 0.f);
-          seed[((slot * 8 + ch) * 4 + jq) * 4 + 2 * hi8 + e] = v;
+        for (int c = lane; c < rk; c += 32) w1 += W[(size_t)c * kD + dm];
+#pragma unroll
+        for (int o = 16; o; o >>= 1) w1 += __shfl_xor_sync(0xffffffffu, w1, o);
+        if (lane < kRopeSeedSlots) {
+          const float mu = pool[hk.mu_off + dm];
+          const float base = rk > 0 ? mu / hk.delta - ((float)(1 << (kb - 1)) - 0.5f) * w1 : 0.f;
+          const int ch = P >> 4, hi8 = (P >> 3) & 1, jq = (P >> 1) & 3, e = P & 1;
+          const float v = rk > 0 ? ldexpf(base, lane + 2 - 10) - w1 : (lane == 0 ? mu : 0.f);
+          seed[((lane * 8 + ch) * 4 + jq) * 4 + 2 * hi8 + e] = v;
         }
       }
     }
-    const unsigned char* qt = a.ws + wh->qt_off + (size_t)it.group * wh->qt_stride;
+    const unsigned char* qt = a.ws + wh->qt_off + (size_t)grp * wh->qt_stride;
     for (int i = tid; i < (int)(decode_qfrag_bytes<G>() / 16); i += blockDim.x)
       reinterpret_cast<uint4*>(qfrag)[i] = reinterpret_cast<const uint4*>(qt + kQtHeaderBytes)[i];
     const float qscale = reinterpret_cast<const float*>(qt)[8];
     __syncthreads();
 
-    // ---- this warp's rows of the item ----
+    // ---- this warp's rows of the group: rows warp, warp + nw, ... (never past the cache's
+    //      rows of a sequence) ----
     const int T = a.seq_lens[gr.seq];
     const int rows_valid = (T + kRowTokens - 1) / kRowTokens;
-    const int row0 = it.row_begin, row1 = min(it.row_end, rows_valid);
+    const int row0 = 0, row1 = min(rows_valid, a.page_table ? 2 * a.pages_per_seq : a.rows_per_seq);
     const uint32_t rbk = rk > 0 ? 16u * rk * kb : 0u, rbv = vr > 0 ? 16u * vr * vb : 0u;
     const uint32_t kst = rk > 0 ? 256u * kb * nk : 0u;  // whole channel tiles (the last may read past the row)
     const bool fits = kst + ((rbv + 127u) & ~127u) <= (uint32_t)ra.stage_bytes;
@@ -555,8 +582,19 @@ __global__ void __launch_bounds__(kRopeMaxWarps * 32, 1) rope_scan_kernel(Decode
       }
     }
     __syncthreads();
-    // ---- merge the warps: m = max m_w, l = sum 2^(m_w - m) l_w, O likewise ----
-    float* part = parts + (size_t)it.slot * pstride;
+    // ---- merge the warps into the group's first slot: m = max m_w, l = sum 2^(m_w - m) l_w,
+    //      O likewise; the group's other slots are left empty (m = -inf, l = 0, O = 0) ----
+    for (int idx = tid; idx < (gr.n_items - 1) * G * (1 + vr); idx += blockDim.x) {
+      const int k = 1 + idx / (G * (1 + vr)), rem = idx % (G * (1 + vr)), g = rem / (1 + vr), e = rem % (1 + vr);
+      float* pg = parts + (size_t)(gr.first_item + k) * pstride + g * gstride;
+      if (e == 0) {
+        pg[0] = -INFINITY;
+        pg[1] = 0.f;
+      } else {
+        pg[3 + e] = 0.f;
+      }
+    }
+    float* part = parts + (size_t)gr.first_item * pstride;
     const size_t wb = rope_warp_bytes<G>(ra.stage_bytes) / sizeof(float);
     const float* mg0 = reinterpret_cast<const float*>(smem + rope_fixed_bytes<G>());
     for (int idx = tid; idx < G * (1 + vr); idx += blockDim.x) {

@@ -86,6 +86,11 @@ def check_plan(L, H, S, caps, r, b):
     runs = [order[0]] + [v for p, v in zip(order, order[1:]) if v != p]
     assert runs == sorted(set(runs))
     assert g[:, 4].max() <= 33
+    # the RoPE decode's staging bound: K row in whole 16-channel tiles + V row (128-aligned)
+    tiles = [256 * (b[hk] if r[hk] else 0) * ((r[hk] + 15) // 16) + (row_bytes(r[hv], b[hv]) + 127) // 128 * 128
+             for (_, _, _, _, _, hk, hv, _) in g]
+    assert info.max_stage_bytes == max(tiles)
+    assert info.max_row_bytes == max(max(row_bytes(r[hk], b[hk]), row_bytes(r[hv], b[hv])) for (*_, hk, hv, _) in g)
     return h, g, it
 
 
