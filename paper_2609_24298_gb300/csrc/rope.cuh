@@ -47,7 +47,7 @@ constexpr int kRopeMaxWarps = 8;
 constexpr int kRopeKTiles = 8;        // channel tiles of 16 (r <= 128)
 constexpr int kRopeSeedSlots = 8;     // windows k = 2 .. 9
 constexpr int kRopeMergeStride = 4 + kD;  // floats per query head in a warp's partial
-constexpr int kRopeCh = 2;            // blocks of 16 positions rebuilt per pass over the codes
+constexpr int kRopeCh = 4;            // blocks of 16 positions rebuilt per pass over the codes
 
 // Table entry of pair j = 4 n + jj within a row: [(jj * 16 + n) * 2 + (0: cos, 1: sin)].  The
 // two pairs (8 ch + jj, 8 ch + 4 + jj) that a lane turns in channel block ch are one float4.
@@ -264,7 +264,7 @@ __device__ __forceinline__ void rope_k_row(const uint8_t* stage, int rk, int cro
       if constexpr (B > 0) {
         // the codes of both token tiles are unpacked again for every kRopeCh blocks of 16
         // positions: holding them for all channel tiles would not fit the registers
-#pragma unroll 1
+#pragma unroll 2
         for (int kt = 0; kt < nk; ++kt) {
           uint32_t wa[B], wb[B];
           load_piece<B>(pa + kt * 8 * 32 * B, wa);
