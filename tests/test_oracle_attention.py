@@ -160,3 +160,17 @@ def test_near_lossless_codes_approach_exact_attention():
     q, ck, cv, pk, pv, xk, xv = setup_decode(T, 128, 2, 128, 2)
     rel2 = np.abs(attention.decode(q, ck, cv, pk, pv) - exact).max() / np.abs(exact).max()
     assert rel2 > rel
+
+
+def test_post_hadamard_channels_are_near_gaussian():
+    """Soft check of Sec. 3.4's Gaussianity argument on the synthetic heads: the median
+    |excess kurtosis| of the rotated channels y = W^T (x - mu) stays below 0.2 (4096 tokens;
+    the estimator's standard deviation is about 0.08)."""
+    src, _ = head(7)
+    x = src.calibration(4096)
+    cal = calibrate.calibrate_head(x)
+    W = calibrate.fuse_basis(cal["U"], 64, synth.hadamard_signs(99, 0, 7, 0))
+    y = compress.project(x, W, cal["mu"])
+    yc = y - y.mean(0)
+    kappa = np.mean(yc ** 4, 0) / np.mean(yc ** 2, 0) ** 2 - 3.0
+    assert np.median(np.abs(kappa)) < 0.2
