@@ -44,6 +44,24 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
+// The dynamic shared memory a kernel may use is granted per device (cudaFuncSetAttribute acts
+// on the current device), so each launch site keeps, per device, the largest size granted.
+constexpr int kMaxDevices = 64;
+using Granted = std::atomic<size_t>[kMaxDevices];
+
+template <typename Kernel>
+cobra_status ensure_smem(Kernel kernel, size_t bytes, Granted& granted) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return COBRA_ECUDA;
+  size_t cur = granted[dev].load(std::memory_order_relaxed);
+  if (bytes <= cur) return COBRA_OK;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes) != cudaSuccess)
+    return COBRA_ECUDA;
+  while (bytes > cur && !granted[dev].compare_exchange_weak(cur, bytes)) {
+  }
+  return COBRA_OK;
+}
+
 }  // namespace
 
 namespace {
@@ -124,13 +142,8 @@ extern "C" cobra_status cobra_compress(const void* params, const cobra_compress_
   int slots[4];
   st = make_x_map(d, x, n_tok, &map, slots);
   if (st != COBRA_OK) return st;
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(compress_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmemBytes) !=
-        cudaSuccess)
-      return COBRA_ECUDA;
-    attr = true;
-  }
+  static Granted granted;
+  if (ensure_smem(compress_tc_kernel, kTcSmemBytes, granted) != COBRA_OK) return COBRA_ECUDA;
   TcArgs a{};
   a.block = static_cast<const unsigned char*>(params);
   a.cache = cache;
@@ -230,13 +243,8 @@ extern "C" cobra_status cobra_append(const void* params, const cobra_compress_de
   cobra_status st = append_args(params, d, x, pos, cache, page_table, a);
   if (st != COBRA_OK) return st;
   const long long grid = (long long)d->n_layers * d->n_kv_heads;  // one CTA per (layer, kv head)
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(append_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)append_smem_bytes()) !=
-        cudaSuccess)
-      return COBRA_ECUDA;
-    attr = true;
-  }
+  static Granted granted;
+  if (ensure_smem(append_kernel, append_smem_bytes(), granted) != COBRA_OK) return COBRA_ECUDA;
   if (launch_pdl(append_kernel, (unsigned)grid, kAppendThreads, append_smem_bytes(), (cudaStream_t)stream, a) !=
       cudaSuccess)
     return COBRA_ECUDA;
@@ -250,15 +258,10 @@ enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 template <int G>
 cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_items, int stages, cudaStream_t s,
                            bool after_plan_kernel = false, const CompressArgs& ak = CompressArgs{}) {
-  static bool head_attr = false;
-  if (!head_attr) {
-    if (cudaFuncSetAttribute(qproj_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)qproj_smem_bytes()) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(combine_kernel<G, kCombineVP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)combine_smem_bytes<kCombineVP>()) != cudaSuccess)
-      return COBRA_ECUDA;
-    head_attr = true;
-  }
+  static Granted qproj_granted, combine_granted;
+  if (ensure_smem(qproj_kernel<G>, qproj_smem_bytes(), qproj_granted) != COBRA_OK ||
+      ensure_smem(combine_kernel<G, kCombineVP>, combine_smem_bytes<kCombineVP>(), combine_granted) != COBRA_OK)
+    return COBRA_ECUDA;
   if (stages & kQproj) {
     // the query projection reads the plan before its wait; right after the plan kernel it is
     // launched in plain stream order
@@ -273,12 +276,8 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
   if (stages & kScan) {
     const size_t smem =
         (size_t)kDecodeWarps * ((size_t)a.ring_bytes + decode_osm_bytes<G>() + decode_qfrag_bytes<G>() + kMaxStages * 8);
-    static size_t attr_set = 0;
-    if (smem > attr_set) {
-      if (cudaFuncSetAttribute(decode_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
-        return COBRA_ECUDA;
-      attr_set = smem;
-    }
+    static Granted granted;
+    if (ensure_smem(decode_kernel<G>, smem, granted) != COBRA_OK) return COBRA_ECUDA;
     int per_sm = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_kernel<G>, kDecodeWarps * 32, smem) != cudaSuccess)
       return COBRA_ECUDA;
@@ -459,13 +458,8 @@ cobra_status launch_rope(const DecodeArgs& a, const RopeArgs& ra0, int n_heads, 
   const int nw = (int)std::min<long long>(kRopeMaxWarps, room > 0 ? room / (long long)per_warp : 0);
   if (nw < 1) return COBRA_EINVAL;  // code rows too large for the staging
   const size_t smem = fixed + (size_t)nw * per_warp;
-  static size_t attr_set = 0;
-  if (smem > attr_set) {
-    if (cudaFuncSetAttribute(rope_scan_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-        cudaSuccess)
-      return COBRA_ECUDA;
-    attr_set = smem;
-  }
+  static Granted granted;
+  if (ensure_smem(rope_scan_kernel<G>, smem, granted) != COBRA_OK) return COBRA_ECUDA;
   if (launch_pdl(rope_qprep_kernel<G>, (unsigned)n_heads, kHeadThreads, 0, s, a, ra) != cudaSuccess)
     return COBRA_ECUDA;
   // one CTA per SM over the groups; the work counter is 0 here (the plan writes it so, every
@@ -539,7 +533,6 @@ namespace {
 constexpr size_t kStaticScratchBytes = COBRA_STATIC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-constexpr int kMaxDevices = 64;
 std::atomic<unsigned char*> g_scratch_ptr[kMaxDevices];
 
 // The host-side address of g_static_scratch on the current device, looked up once per device.
@@ -746,13 +739,8 @@ extern "C" cobra_status cobra_calibrate_heads(int n_heads, int n_tok, const floa
   if (!aligned(x, 4) || (q && !aligned(q, 4)) || !aligned(mu, 8) || !aligned(lam, 8) || !aligned(U, 8) ||
       !aligned(w, 8))
     return COBRA_EALIGN;
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(calib_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)calib_smem_bytes()) !=
-        cudaSuccess)
-      return COBRA_ECUDA;
-    attr = true;
-  }
+  static Granted granted;
+  if (ensure_smem(calib_kernel, calib_smem_bytes(), granted) != COBRA_OK) return COBRA_ECUDA;
   CalibArgs a{};
   a.x = x;
   a.q = n_q > 0 ? q : nullptr;
