@@ -198,6 +198,23 @@ cobra_status cobra_params_build(void* dev_block, size_t block_bytes, int n_heads
                                 const float* delta, const uint64_t* cache_off, const float* W_all,
                                 const float* mu_all, void* stream);
 
+/* The same block built in host memory (`image`, >= cobra_params_bytes bytes; same inputs as
+ * cobra_params_build): the bytes the device block holds, with an FNV-1a 64 checksum in the
+ * header.  This is the checkpoint of a calibration (Table alg:kvrobin step 6 stores it once
+ * per model): write it to a file, read it back, and upload it with cobra_params_upload. */
+cobra_status cobra_params_image(void* image, size_t image_bytes, int n_heads, const int* r, const int* b,
+                                const float* delta, const uint64_t* cache_off, const float* W_all,
+                                const float* mu_all);
+
+/* Check a host image: magic, version, sizes (image_bytes must equal the block's size), every
+ * head's fields and offsets, and the checksum.  COBRA_OK, else COBRA_EINVAL. */
+cobra_status cobra_params_verify(const void* image, size_t image_bytes);
+
+/* Verify a host image, then copy it into caller-allocated device memory (256-byte aligned,
+ * >= image_bytes) with cudaMemcpyAsync on `stream`; the call synchronises the stream. */
+cobra_status cobra_params_upload(void* dev_block, size_t block_bytes, const void* image, size_t image_bytes,
+                                 void* stream);
+
 /* ---------------------------------------------------------------------------------------
  * Compression (device).  Table alg:kvrobin step 7: z_t = quantize(W^T (x_t - mu), b*) with
  * the projection and Hadamard as one multiply (Sec. 3.4), packed into the cache (step 8).

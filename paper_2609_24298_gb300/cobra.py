@@ -72,6 +72,9 @@ SIGNATURES = {
     "cobra_params_bytes": (c_int, [c_int, P_int, P_size]),
     "cobra_params_build": (c_int, [c_void_p, c_size_t, c_int, P_int, P_int, P_float, P_u64, P_float, P_float,
                                    c_void_p]),
+    "cobra_params_image": (c_int, [c_void_p, c_size_t, c_int, P_int, P_int, P_float, P_u64, P_float, P_float]),
+    "cobra_params_verify": (c_int, [c_void_p, c_size_t]),
+    "cobra_params_upload": (c_int, [c_void_p, c_size_t, c_void_p, c_size_t, c_void_p]),
     "cobra_compress": (c_int, [c_void_p, ctypes.POINTER(CompressDesc), c_void_p, c_int, c_int, c_void_p, c_void_p,
                                c_void_p]),
     "cobra_append": (c_int, [c_void_p, ctypes.POINTER(CompressDesc), c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
@@ -302,6 +305,35 @@ def cobra_params_build(dev_block, nbytes: int, r, b, delta, cache_off, W_list, m
     mu, mp = _np(mu_all, np.float32, ctypes.c_float)
     st = lib().cobra_params_build(_ptr(dev_block), int(nbytes), len(r), rp, bp, dp, op, Wp, mp, _stream(stream))
     _chk("cobra_params_build", st)
+
+
+def cobra_params_image(r, b, delta, cache_off, W_list, mu_all) -> np.ndarray:
+    """The parameter block as host bytes (uint8), with its checksum: a calibration checkpoint."""
+    r, rp = _np(r, np.int32, c_int)
+    b, bp = _np(b, np.int32, c_int)
+    delta, dp = _np(delta, np.float32, ctypes.c_float)
+    offs, op = _np(cache_off, np.uint64, ctypes.c_uint64)
+    cols = [np.asarray(W, np.float32).T.reshape(-1) for W in W_list]  # column-major per head
+    Wall = np.concatenate(cols) if cols else np.zeros(1, np.float32)
+    Wall, Wp = _np(Wall if Wall.size else np.zeros(1, np.float32), np.float32, ctypes.c_float)
+    mu, mp = _np(mu_all, np.float32, ctypes.c_float)
+    img = np.zeros(cobra_params_bytes(r), np.uint8)
+    st = lib().cobra_params_image(img.ctypes.data_as(c_void_p), img.nbytes, len(r), rp, bp, dp, op, Wp, mp)
+    _chk("cobra_params_image", st)
+    return img
+
+
+def cobra_params_verify(image) -> int:
+    """Status of a host image check (does not raise): COBRA_OK or COBRA_EINVAL."""
+    img = np.ascontiguousarray(image, np.uint8)
+    return lib().cobra_params_verify(img.ctypes.data_as(c_void_p), img.nbytes)
+
+
+def cobra_params_upload(dev_block, nbytes: int, image, stream=None):
+    img = np.ascontiguousarray(image, np.uint8)
+    st = lib().cobra_params_upload(_ptr(dev_block), int(nbytes), img.ctypes.data_as(c_void_p), img.nbytes,
+                                   _stream(stream))
+    _chk("cobra_params_upload", st)
 
 
 def compress_desc(**kw) -> CompressDesc:

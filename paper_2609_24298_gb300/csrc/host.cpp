@@ -6,6 +6,7 @@
 // file is compiled without FMA contraction, so the allocator's results are reproducible
 // bit for bit by any implementation that follows the same order.
 #include <algorithm>
+#include <cstddef>
 #include <cmath>
 #include <cstring>
 #include <limits>
@@ -662,15 +663,26 @@ extern "C" cobra_status cobra_params_bytes(int n_heads, const int* r, size_t* by
   return COBRA_OK;
 }
 
-extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, int n_heads, const int* r, const int* b,
-                                           const float* delta, const uint64_t* cache_off, const float* W_all,
-                                           const float* mu_all, void* stream) {
+namespace {
+// 64-bit FNV-1a (Fowler-Noll-Vo) over the block, its checksum field taken as zero
+uint64_t block_checksum(const unsigned char* p, size_t n) {
+  uint64_t h = 14695981039346656037ull;
+  const size_t cs = offsetof(cobra::BlockHeader, checksum);
+  for (size_t i = 0; i < n; ++i) {
+    const unsigned char c = (i >= cs && i < cs + sizeof(uint64_t)) ? 0 : p[i];
+    h = (h ^ c) * 1099511628211ull;
+  }
+  return h;
+}
+
+// The block's bytes in host memory (what the device block holds), with its checksum.
+cobra_status build_block_image(std::vector<unsigned char>& img, int n_heads, const int* r, const int* b,
+                               const float* delta, const uint64_t* cache_off, const float* W_all,
+                               const float* mu_all) {
   size_t need = 0;
   cobra_status st = cobra_params_bytes(n_heads, r, &need);
   if (st != COBRA_OK) return st;
-  if (!dev_block || !b || !delta || !cache_off || !mu_all) return COBRA_EINVAL;
-  if (block_bytes < need) return COBRA_ESPACE;
-  if (((uintptr_t)dev_block) & 255) return COBRA_EALIGN;
+  if (!b || !delta || !cache_off || !mu_all) return COBRA_EINVAL;
   size_t total_r = 0;
   for (int h = 0; h < n_heads; ++h) {
     if (r[h] > 0 && (b[h] < 1 || b[h] > 8 || !(delta[h] > 0.0f) || !std::isfinite(delta[h]))) return COBRA_EINVAL;
@@ -678,7 +690,7 @@ extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, 
     total_r += r[h];
   }
   if (total_r > 0 && !W_all) return COBRA_EINVAL;
-  std::vector<unsigned char> img(need, 0);
+  img.assign(need, 0);
   auto* hdr = reinterpret_cast<cobra::BlockHeader*>(img.data());
   hdr->magic = cobra::kBlockMagic;
   hdr->version = COBRA_VERSION;
@@ -716,10 +728,89 @@ extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, 
     f += r[h];
     wsrc += (size_t)d * r[h];
   }
+  hdr->checksum = block_checksum(img.data(), img.size());
+  return COBRA_OK;
+}
+
+cobra_status upload_block(void* dev_block, size_t block_bytes, const void* image, size_t bytes, void* stream) {
+  if (!dev_block) return COBRA_EINVAL;
+  if (block_bytes < bytes) return COBRA_ESPACE;
+  if (((uintptr_t)dev_block) & 255) return COBRA_EALIGN;
   cudaStream_t s = (cudaStream_t)stream;
-  if (cudaMemcpyAsync(dev_block, img.data(), need, cudaMemcpyHostToDevice, s) != cudaSuccess) return COBRA_ECUDA;
+  if (cudaMemcpyAsync(dev_block, image, bytes, cudaMemcpyHostToDevice, s) != cudaSuccess) return COBRA_ECUDA;
   if (cudaStreamSynchronize(s) != cudaSuccess) return COBRA_ECUDA;
   return COBRA_OK;
+}
+}  // namespace
+
+extern "C" cobra_status cobra_params_build(void* dev_block, size_t block_bytes, int n_heads, const int* r, const int* b,
+                                           const float* delta, const uint64_t* cache_off, const float* W_all,
+                                           const float* mu_all, void* stream) {
+  size_t need = 0;
+  cobra_status st = cobra_params_bytes(n_heads, r, &need);
+  if (st != COBRA_OK) return st;
+  if (!dev_block || !b || !delta || !cache_off || !mu_all) return COBRA_EINVAL;
+  if (block_bytes < need) return COBRA_ESPACE;
+  if (((uintptr_t)dev_block) & 255) return COBRA_EALIGN;
+  std::vector<unsigned char> img;
+  st = build_block_image(img, n_heads, r, b, delta, cache_off, W_all, mu_all);
+  if (st != COBRA_OK) return st;
+  return upload_block(dev_block, block_bytes, img.data(), img.size(), stream);
+}
+
+extern "C" cobra_status cobra_params_image(void* image, size_t image_bytes, int n_heads, const int* r, const int* b,
+                                           const float* delta, const uint64_t* cache_off, const float* W_all,
+                                           const float* mu_all) {
+  size_t need = 0;
+  cobra_status st = cobra_params_bytes(n_heads, r, &need);
+  if (st != COBRA_OK) return st;
+  if (!image) return COBRA_EINVAL;
+  if (image_bytes < need) return COBRA_ESPACE;
+  std::vector<unsigned char> img;
+  st = build_block_image(img, n_heads, r, b, delta, cache_off, W_all, mu_all);
+  if (st != COBRA_OK) return st;
+  std::memcpy(image, img.data(), img.size());
+  return COBRA_OK;
+}
+
+extern "C" cobra_status cobra_params_verify(const void* image, size_t image_bytes) {
+  if (!image || image_bytes < sizeof(cobra::BlockHeader)) return COBRA_EINVAL;
+  const auto* p = static_cast<const unsigned char*>(image);
+  cobra::BlockHeader hdr;
+  std::memcpy(&hdr, p, sizeof(hdr));
+  if (hdr.magic != cobra::kBlockMagic || hdr.version != COBRA_VERSION || hdr.d != cobra::kD || hdr.n_heads < 1 ||
+      hdr.n_heads > (1 << 20) || hdr.heads_off != sizeof(cobra::BlockHeader))
+    return COBRA_EINVAL;
+  const size_t n = (size_t)hdr.n_heads;
+  if (hdr.pool_off != align_up(hdr.heads_off + sizeof(cobra::HeadEntry) * n, 256) || hdr.pool_off > image_bytes)
+    return COBRA_EINVAL;
+  std::vector<int> r(n);
+  for (size_t h = 0; h < n; ++h) {
+    cobra::HeadEntry e;
+    std::memcpy(&e, p + hdr.heads_off + h * sizeof(e), sizeof(e));
+    r[h] = e.r;
+    if (e.r < 0 || e.r > cobra::kD || (e.r & 1)) return COBRA_EINVAL;
+  }
+  size_t need = 0;
+  if (cobra_params_bytes((int)n, r.data(), &need) != COBRA_OK || need != image_bytes ||
+      hdr.pool_floats != pool_floats_for((int)n, r.data()))
+    return COBRA_EINVAL;
+  for (size_t h = 0; h < n; ++h) {
+    cobra::HeadEntry e;
+    std::memcpy(&e, p + hdr.heads_off + h * sizeof(e), sizeof(e));
+    if (e.r > 0 && (e.b < 1 || e.b > 8 || !(e.delta > 0.0f))) return COBRA_EINVAL;
+    if (e.w_off + (uint64_t)cobra::kD * e.r > hdr.pool_floats || e.mu_off + cobra::kD > hdr.pool_floats ||
+        e.wmu_off + (uint64_t)e.r > hdr.pool_floats || (e.cache_off & 255))
+      return COBRA_EINVAL;
+  }
+  return block_checksum(p, image_bytes) == hdr.checksum ? COBRA_OK : COBRA_EINVAL;
+}
+
+extern "C" cobra_status cobra_params_upload(void* dev_block, size_t block_bytes, const void* image, size_t image_bytes,
+                                            void* stream) {
+  const cobra_status st = cobra_params_verify(image, image_bytes);
+  if (st != COBRA_OK) return st;
+  return upload_block(dev_block, block_bytes, image, image_bytes, stream);
 }
 
 // ----------------------------------------------------------------------------------------

@@ -21,7 +21,8 @@ struct BlockHeader {
   uint64_t heads_off;    // bytes from block start
   uint64_t pool_off;     // bytes from block start
   uint64_t pool_floats;
-  uint64_t reserved[3];
+  uint64_t checksum;     // FNV-1a 64 of the whole block with this field zero
+  uint64_t reserved[2];
 };
 static_assert(sizeof(BlockHeader) == 64, "header size");
 
