@@ -18,6 +18,7 @@ Modules
   attention  dequantise-on-read decode attention, plain definition and rank-space algebra
   rope       decode with the rotary embedding applied to the reconstructed keys and the query
   compress   per-token projection + quantisation (Table alg:kvrobin step 7)
+  measured   App. E's measured per-head distortion tables and the exact DP over them
 
 Parity status: the damped C2 update is a heuristic with no optimality guarantee
 (App. D says so itself); its output is pinned only through invariants - "parity unpinned"
