@@ -614,6 +614,14 @@ def run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out, cpu_ba
             "gpu_launches": 3 * K}
 
 
+def aux_leg(fn, *a):
+    """The JSON object of a leg measured after the headline, or {"error": ...} if it failed."""
+    try:
+        return fn(*a)
+    except Exception as e:  # the headline line is printed either way
+        return {"error": f"{type(e).__name__}: {e}"[:400]}
+
+
 def run_cobra(args):
     import torch
     import torch.distributed as dist
@@ -798,20 +806,21 @@ def run_cobra(args):
 
     peak, peak_kind = hbm_peak()
     achieved = bytes_step / (scan_ms * 1e-3) / 1e9
+    # the legs below are measured after the headline: a failure in one is reported in its place
     calibration = None
     if not args.no_calibration and rank == 0:
-        calibration = run_calibration_leg(args, dev, stream, srcs, not args.no_cpu_baseline and world == 1)
+        calibration = aux_leg(run_calibration_leg, args, dev, stream, srcs, not args.no_cpu_baseline and world == 1)
     measured = None
     if not args.no_measured and rank == 0:
-        measured = run_measured_leg(args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
+        measured = aux_leg(run_measured_leg, args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
     rope = None
     if not args.no_rope and rank == 0:
-        rope = run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out,
-                            not args.no_cpu_baseline and world == 1)
+        rope = aux_leg(run_rope_leg, args, dev, stream, hp, wl, desc, ws, info, q, lens, out,
+                       not args.no_cpu_baseline and world == 1)
     compress = None
     if not args.no_compress:
         del hin, hout
-        compress = run_compress_leg(args, dev, stream, peak)
+        compress = aux_leg(run_compress_leg, args, dev, stream, peak)
     traffic = profiled_traffic()
     if rank == 0:
         line = {
