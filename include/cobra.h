@@ -118,14 +118,16 @@ cobra_status cobra_calibrate_heads(int n_heads, int n_tok, const float* x, int n
  * and D[h][i][j] = (1/n_tok) sum_t sum_k omega_k (u_k . (x_t - x^_t))^2 is written in fp64,
  * omega_k = 1 for the MSE objective or sigma_Q,k^2 for attention-KL, so that r = 0 gives
  * sum_k w_k.  Device inputs, per head h and d = 128: x [n_heads][n_tok][d] fp32 tokens; U
- * [n_heads][d*d] fp32, column k = u_k in the allocator's order; lam [n_heads][d] fp64
- * eigenvalues in the same order; omega, mu [n_heads][d] fp32; signs [n_heads][d] int8 (+1/-1).
+ * [n_heads][d*d] fp32, column k = u_k in the allocator's order; lam, w [n_heads][d] fp64
+ * eigenvalues and allocator weights in the same order (cobra_calibrate_heads' outputs: w =
+ * lambda for MSE, sigma_Q^2 lambda for attention-KL), from which the library takes omega_k =
+ * w_k / lambda_k (0 where lambda_k = 0); mu [n_heads][d] fp32; signs [n_heads][d] int8 (+1/-1).
  * coords: device workspace of n_heads * n_tok * d floats (overwritten).  Host lists: r_list
  * (1..65 entries) strictly ascending in [0, 128], b_list (1..16 entries) in [1, 8].  Two
  * launches; nothing is synchronised.  Errors: EINVAL, EALIGN (4-byte floats, 8-byte
  * doubles), ECUDA. */
 cobra_status cobra_measure_distortion(int n_heads, int n_tok, const float* x, const float* U, const double* lam,
-                                      const float* omega, const float* mu, const int8_t* signs, int n_r,
+                                      const double* w, const float* mu, const int8_t* signs, int n_r,
                                       const int* r_list, int n_b, const int* b_list, float* coords, double* D,
                                       void* stream);
 
@@ -395,7 +397,11 @@ cobra_status cobra_decode_rope_attn(const void* params, const cobra_decode_desc*
  *   - Returns COBRA_ESPACE when seqs x layers x kv heads chunks do not fit the array
  *     (about 6.4 KB per chunk for group 4, 8.5 KB for group 8).
  *   - The first call on each device looks up the array's address on that device (with the
- *     device current); make that first call before any stream capture.
+ *     device current); make that first call before any stream capture.  The address is
+ *     looked up again when the current context on the device changes (after cudaDeviceReset,
+ *     or with another context made current), so such a call also comes before any capture.
+ *   - A descriptor naming a head the parameter block does not hold is reported by cobra_check
+ *     (COBRA_EINVAL); that (seq, layer, kv head) is then computed over no tokens.
  *   - All calls on a device share the one array and it keeps the last call's contents: calls
  *     that can overlap on the GPU (different streams, no ordering between them) race and must
  *     not be issued.

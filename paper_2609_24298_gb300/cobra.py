@@ -218,13 +218,14 @@ def cobra_calibrate_heads(x, q, mu, lam, U, w, stream=None):
     _chk("cobra_calibrate_heads", st)
 
 
-def cobra_measure_distortion(x, U, lam, omega, mu, signs, r_list, b_list, coords, D, stream=None):
+def cobra_measure_distortion(x, U, lam, w, mu, signs, r_list, b_list, coords, D, stream=None):
     """Measured distortion tables on the device (App. E); all array arguments are device
-    tensors except the two host lists."""
+    tensors except the two host lists.  lam and w are the calibration's eigenvalues and
+    allocator weights (fp64); the library derives the error weights from them."""
     rl, rlp = _np(r_list, np.int32, c_int)
     bl, blp = _np(b_list, np.int32, c_int)
     n_heads, n_tok = int(x.shape[0]), int(x.shape[1])
-    st = lib().cobra_measure_distortion(n_heads, n_tok, _ptr(x), _ptr(U), _ptr(lam), _ptr(omega), _ptr(mu),
+    st = lib().cobra_measure_distortion(n_heads, n_tok, _ptr(x), _ptr(U), _ptr(lam), _ptr(w), _ptr(mu),
                                         _ptr(signs), len(rl), rlp, len(bl), blp, _ptr(coords), _ptr(D),
                                         _stream(stream))
     _chk("cobra_measure_distortion", st)

@@ -798,7 +798,15 @@ extern "C" cobra_status cobra_params_verify(const void* image, size_t image_byte
   for (size_t h = 0; h < n; ++h) {
     cobra::HeadEntry e;
     std::memcpy(&e, p + hdr.heads_off + h * sizeof(e), sizeof(e));
-    if (e.r > 0 && (e.b < 1 || e.b > 8 || !(e.delta > 0.0f))) return COBRA_EINVAL;
+    // the same head fields cobra_params_build writes: for r > 0 a finite positive step and its
+    // reciprocal rounded from double, bit for bit; for r = 0 zeros
+    if (e.r > 0) {
+      if (e.b < 1 || e.b > 8 || !(e.delta > 0.0f) || !std::isfinite(e.delta)) return COBRA_EINVAL;
+      const float inv = (float)(1.0 / (double)e.delta);
+      if (std::memcmp(&inv, &e.inv_delta, sizeof(float)) != 0) return COBRA_EINVAL;
+    } else if (e.b != 0 || e.delta != 0.0f || e.inv_delta != 0.0f) {
+      return COBRA_EINVAL;
+    }
     if (e.w_off + (uint64_t)cobra::kD * e.r > hdr.pool_floats || e.mu_off + cobra::kD > hdr.pool_floats ||
         e.wmu_off + (uint64_t)e.r > hdr.pool_floats || (e.cache_off & 255))
       return COBRA_EINVAL;

@@ -533,20 +533,48 @@ namespace {
 constexpr size_t kStaticScratchBytes = COBRA_STATIC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-std::atomic<unsigned char*> g_scratch_ptr[kMaxDevices];
+// Address of g_static_scratch per device, with the context it was looked up in: a device
+// reset (cudaDeviceReset) or another context made current on the device gives the array a new
+// address, so the lookup is repeated whenever the current context differs from the recorded one.
+struct ScratchAddr {
+  std::atomic<unsigned char*> ptr{nullptr};
+  std::atomic<void*> ctx{nullptr};
+};
+ScratchAddr g_scratch_addr[kMaxDevices];
 
-// The host-side address of g_static_scratch on the current device, looked up once per device.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+CtxGetCurrentFn ctx_get_current() {
+  static CtxGetCurrentFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(p);
+  }
+  return fn;
+}
+
+// The host-side address of g_static_scratch on the current device (looked up with that device
+// and context current; cudaGetSymbolAddress allocates nothing).
 cobra_status static_scratch(unsigned char** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return COBRA_ECUDA;
-  unsigned char* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
-  if (!p) {
-    void* addr = nullptr;
-    if (cudaGetSymbolAddress(&addr, g_static_scratch) != cudaSuccess || !addr) return COBRA_ECUDA;
-    p = static_cast<unsigned char*>(addr);
-    g_scratch_ptr[dev].store(p, std::memory_order_release);
+  CtxGetCurrentFn get = ctx_get_current();
+  CUcontext ctx = nullptr;
+  ScratchAddr& slot = g_scratch_addr[dev];
+  unsigned char* p = slot.ptr.load(std::memory_order_acquire);
+  if (p && get && get(&ctx) == CUDA_SUCCESS && ctx == slot.ctx.load(std::memory_order_acquire)) {
+    *out = p;
+    return COBRA_OK;
   }
-  *out = p;
+  void* addr = nullptr;
+  if (cudaGetSymbolAddress(&addr, g_static_scratch) != cudaSuccess || !addr) return COBRA_ECUDA;
+  ctx = nullptr;
+  if (get) get(&ctx);
+  slot.ctx.store(ctx, std::memory_order_release);
+  slot.ptr.store(static_cast<unsigned char*>(addr), std::memory_order_release);
+  *out = static_cast<unsigned char*>(addr);
   return COBRA_OK;
 }
 
@@ -582,14 +610,22 @@ __global__ void static_plan_kernel(unsigned char* ws, const unsigned char* block
   WsGroup* groups = reinterpret_cast<WsGroup*>(ws + z.groups_off);
   WsItem* items = reinterpret_cast<WsItem*>(ws + z.items_off);
   int* hg = reinterpret_cast<int*>(ws + z.hg_off);
-  const HeadEntry* heads = head_table(block);
+  const int n_heads = reinterpret_cast<const BlockHeader*>(block)->n_heads;
   for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < n_groups; g += gridDim.x * blockDim.x) {
     const int h = g % d.n_kv_heads, l = (g / d.n_kv_heads) % d.n_layers, s = g / (d.n_kv_heads * d.n_layers);
-    const int hk = d.k_head0 + l * d.layer_stride + h, hv = d.v_head0 + l * d.layer_stride + h;
+    int hk = d.k_head0 + l * d.layer_stride + h, hv = d.v_head0 + l * d.layer_stride + h;
+    int rows = cap_rows;
+    if (hk >= n_heads || hv >= n_heads) {
+      // the descriptor names a head the parameter block does not have: report it (cobra_check
+      // returns COBRA_EINVAL) and plan an empty chunk on head 0, so nothing reads past the
+      // head table or the cache
+      atomicOr(&g_status, 2u);
+      hk = hv = 0;
+      rows = 0;
+    }
     groups[g] = WsGroup{s, l, h, g, 1, hk, hv, 0};
-    items[g] = WsItem{g, 0, cap_rows, g};
+    items[g] = WsItem{g, 0, rows, g};
     hg[((size_t)l * d.n_kv_heads + h) * d.n_seqs + s] = g;
-    (void)heads;
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) {
     WsHeader hd;
@@ -694,20 +730,20 @@ extern "C" cobra_status cobra_check(void* stream) {
 }
 
 extern "C" cobra_status cobra_measure_distortion(int n_heads, int n_tok, const float* x, const float* U,
-                                                 const double* lam, const float* omega, const float* mu,
+                                                 const double* lam, const double* w, const float* mu,
                                                  const int8_t* signs, int n_r, const int* r_list, int n_b,
                                                  const int* b_list, float* coords, double* D, void* stream) {
-  if (n_heads < 1 || n_heads > 65535 || n_tok < 1 || !x || !U || !lam || !omega || !mu || !signs || !r_list ||
+  if (n_heads < 1 || n_heads > 65535 || n_tok < 1 || !x || !U || !lam || !w || !mu || !signs || !r_list ||
       !b_list || !coords || !D || n_r < 1 || n_r > kMeasureMaxR || n_b < 1 || n_b > kMeasureMaxB)
     return COBRA_EINVAL;
-  if (!aligned(x, 4) || !aligned(U, 4) || !aligned(lam, 8) || !aligned(omega, 4) || !aligned(mu, 4) ||
+  if (!aligned(x, 4) || !aligned(U, 4) || !aligned(lam, 8) || !aligned(w, 8) || !aligned(mu, 4) ||
       !aligned(coords, 4) || !aligned(D, 8))
     return COBRA_EALIGN;
   MeasureArgs a{};
   a.x = x;
   a.U = U;
   a.lam = lam;
-  a.omega = omega;
+  a.w = w;
   a.mu = mu;
   a.signs = signs;
   a.coords = coords;

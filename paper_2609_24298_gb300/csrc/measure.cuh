@@ -27,7 +27,7 @@ struct MeasureArgs {
   const float* x;        // [n_heads][n_tok][kD] calibration tokens
   const float* U;        // [n_heads][kD * kD] basis, column k = u_k (allocator order)
   const double* lam;     // [n_heads][kD] eigenvalues in the same order
-  const float* omega;    // [n_heads][kD] error weight per direction
+  const double* w;       // [n_heads][kD] allocator weights in the same order (lambda or sigma_Q^2 lambda)
   const float* mu;       // [n_heads][kD]
   const int8_t* signs;   // [n_heads][kD] Hadamard column signs
   float* coords;         // [n_heads][n_tok][kD] workspace: c = (x - mu) U
@@ -110,7 +110,8 @@ __global__ void __launch_bounds__(256) measure_kernel(MeasureArgs a) {
   int bs[4];
   float sg[4], om[4], inv[4];
   const int8_t* s = a.signs + (size_t)h * kD;
-  const float* omega = a.omega + (size_t)h * kD;
+  const double* wt = a.w + (size_t)h * kD;
+  const double* lam = a.lam + (size_t)h * kD;
 #pragma unroll
   for (int m = 0; m < 4; ++m) {
     const int k = lane + 32 * m;
@@ -122,7 +123,8 @@ __global__ void __launch_bounds__(256) measure_kernel(MeasureArgs a) {
       }
     bs[m] = size;  // 0 past r
     sg[m] = k < r ? (float)s[k] : 0.f;
-    om[m] = omega[k];
+    // error weight omega_k = w_k / lambda_k: 1 for the MSE objective, sigma_Q,k^2 for attention-KL
+    om[m] = lam[k] > 0.0 ? (float)(wt[k] / lam[k]) : 0.f;
     inv[m] = size > 0 ? rsqrtf((float)size) : 0.f;
   }
   // with unit weights (the MSE objective) the rotation back preserves the norm: the error is

@@ -148,27 +148,21 @@ def calibrate_heads_device(xs, qs=None, device="cuda"):
     return out
 
 
-def error_weights(cal) -> np.ndarray:
-    """omega_k = w_k / lambda_k: 1 for the MSE objective, sigma_Q,k^2 for attention-KL (0 on a
-    direction without variance)."""
-    lam = np.asarray(cal["lam"], np.float64)
-    return np.where(lam > 0, np.asarray(cal["w"], np.float64) / np.where(lam > 0, lam, 1.0), 0.0)
-
-
 def measured_tables(cals, srcs, r_list, b_list, device="cuda", n_tok: int = 512, stream=None) -> np.ndarray:
     """App. E: every head's calibration tokens through the deployed quantizer at every
     candidate (r, b), on the device (cobra_measure_distortion).  Returns D [n][len(r)][len(b)]."""
     f32 = lambda a: torch.tensor(np.asarray(a, np.float32), device=device).contiguous()
     x = f32(np.stack([s.calibration(n_tok) for s in srcs]))
     U = f32(np.stack([c["U"].T.reshape(-1) for c in cals]))  # column k of U = row k of U^T
-    lam = torch.tensor(np.stack([c["lam"] for c in cals]), dtype=torch.float64, device=device).contiguous()
-    omega = f32(np.stack([error_weights(c) for c in cals]))
+    f64 = lambda a: torch.tensor(np.asarray(a, np.float64), device=device).contiguous()
+    lam = f64(np.stack([c["lam"] for c in cals]))
+    w = f64(np.stack([c["w"] for c in cals]))
     mu = f32(np.stack([c["mu"] for c in cals]))
     signs = torch.tensor(np.stack([synth.hadamard_signs(*s.key) for s in srcs]), dtype=torch.int8,
                          device=device).contiguous()
     coords = torch.empty((len(cals), n_tok, D), dtype=torch.float32, device=device)
     out = torch.empty((len(cals), len(r_list), len(b_list)), dtype=torch.float64, device=device)
-    cobra.cobra_measure_distortion(x, U, lam, omega, mu, signs, r_list, b_list, coords, out, stream)
+    cobra.cobra_measure_distortion(x, U, lam, w, mu, signs, r_list, b_list, coords, out, stream)
     torch.cuda.synchronize()
     return out.cpu().numpy()
 

@@ -71,13 +71,14 @@ def device_tables(hs, rg, bg):
     f32 = lambda a: torch.tensor(np.stack(a), dtype=torch.float32, device=DEV).contiguous()
     x = f32([h[0] for h in hs])
     U = f32([h[1]["U"].T.reshape(-1) for h in hs])  # row k of U^T = column k of U
-    lam = torch.tensor(np.stack([h[1]["lam"] for h in hs]), dtype=torch.float64, device=DEV).contiguous()
-    omega = f32([h[2] for h in hs])
+    f64 = lambda a: torch.tensor(np.stack(a), dtype=torch.float64, device=DEV).contiguous()
+    lam = f64([h[1]["lam"] for h in hs])
+    w = f64([h[1]["w"] for h in hs])
     mu = f32([h[1]["mu"] for h in hs])
     signs = torch.tensor(np.stack([h[3] for h in hs]), dtype=torch.int8, device=DEV).contiguous()
     coords = torch.empty((len(hs), x.shape[1], 128), dtype=torch.float32, device=DEV)
     D = torch.full((len(hs), len(rg), len(bg)), float("nan"), dtype=torch.float64, device=DEV)
-    cobra.cobra_measure_distortion(x, U, lam, omega, mu, signs, rg, bg, coords, D)
+    cobra.cobra_measure_distortion(x, U, lam, w, mu, signs, rg, bg, coords, D)
     torch.cuda.synchronize()
     return D.cpu().numpy()
 

@@ -92,3 +92,40 @@ def test_corrupt_images_are_rejected():
     with pytest.raises(cobra.CobraError) as e:
         cobra.cobra_params_upload(256, n, img[:-4])
     assert e.value.status == cobra.COBRA_EINVAL
+
+
+def resign(raw: bytearray) -> np.ndarray:
+    """The image with its header checksum recomputed (so that only the field checks can reject it)."""
+    raw[40:48] = bytes(8)
+    raw[40:48] = struct.pack("<Q", fnv1a64(bytes(raw)))
+    return np.frombuffer(bytes(raw), np.uint8)
+
+
+@pytest.mark.parametrize("field", ["delta_inf", "delta_nan", "inv_delta", "r0_b", "r0_delta", "r0_inv"])
+def test_inconsistent_head_fields_are_rejected_with_a_valid_checksum(field):
+    """A checkpoint written by another tool with a correct checksum is still checked field by
+    field, as strictly as the build path: a finite step, its reciprocal as the build rounds it,
+    and zeros in the quantiser fields of a head without codes (Sec. 3, static scalar quantizer)."""
+    img = image()[0]
+    raw = bytearray(img.tobytes())
+    heads_off = 64
+    h_codes, h_empty = 0, 1  # rb = [(64, 2), (0, 1), ...]
+    base = heads_off + 64 * h_codes
+    if field == "delta_inf":
+        struct.pack_into("<f", raw, base + 8, float("inf"))
+        struct.pack_into("<f", raw, base + 12, 0.0)
+    elif field == "delta_nan":
+        struct.pack_into("<f", raw, base + 8, float("nan"))
+    elif field == "inv_delta":
+        inv = struct.unpack_from("<I", raw, base + 12)[0]
+        struct.pack_into("<I", raw, base + 12, inv + 1)  # one ulp off
+    else:
+        e = heads_off + 64 * h_empty
+        off = {"r0_b": 4, "r0_delta": 8, "r0_inv": 12}[field]
+        if field == "r0_b":
+            struct.pack_into("<i", raw, e + off, 3)
+        else:
+            struct.pack_into("<f", raw, e + off, 0.5)
+    good = resign(bytearray(img.tobytes()))
+    assert cobra.cobra_params_verify(good) == cobra.COBRA_OK  # re-signing alone keeps it valid
+    assert cobra.cobra_params_verify(resign(raw)) == cobra.COBRA_EINVAL
