@@ -264,7 +264,8 @@ def run_reference(args):
     el = time.perf_counter() - t0
     gbs = sample.bytes * args.steps / el / 1e9
     desc = (f"one (seq, layer, kv-head) group per step: decode over {T} tokens with K and V at r={SAMPLE_R}, "
-            f"b={SAMPLE_B} + append-compress of the new token (fp64 numpy)")
+            f"b={SAMPLE_B} + append-compress of the new token (fp64 numpy); a fixed-allocation sample: at 1 bpd "
+            "every head stores r b = 128 bits per token, the same bytes as the allocated heads, whose (r, b) vary")
     out = {"metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": args.gpus, "steps": args.steps,
            "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
@@ -482,8 +483,7 @@ def run_measured_leg(args, dev, stream, cals, srcs, cpu_baseline: bool):
     x = f32(xs)
     U = f32(np.stack([c["U"].T.reshape(-1) for c in cals]))
     lam = torch.tensor(np.stack([c["lam"] for c in cals]), dtype=torch.float64, device=dev).contiguous()
-    om = np.stack([np.where(c["lam"] > 0, c["w"] / np.where(c["lam"] > 0, c["lam"], 1.0), 0.0) for c in cals])
-    omega = f32(om)
+    w = torch.tensor(np.stack([c["w"] for c in cals]), dtype=torch.float64, device=dev).contiguous()
     mu = f32(np.stack([c["mu"] for c in cals]))
     signs = torch.tensor(np.stack([synth.hadamard_signs(*s.key) for s in srcs]), dtype=torch.int8,
                          device=dev).contiguous()
@@ -492,7 +492,7 @@ def run_measured_leg(args, dev, stream, cals, srcs, cpu_baseline: bool):
     D = torch.empty((n, len(rg), len(bg)), dtype=torch.float64, device=dev)
 
     def call():
-        cobra.cobra_measure_distortion(x, U, lam, omega, mu, signs, rg, bg, coords, D, stream)
+        cobra.cobra_measure_distortion(x, U, lam, w, mu, signs, rg, bg, coords, D, stream)
 
     for _ in range(2):
         call()
@@ -530,7 +530,7 @@ def run_measured_leg(args, dev, stream, cals, srcs, cpu_baseline: bool):
         out["cpu_baseline"] = {"value": el * n * 1e3, "unit": "ms per table set", "cores": cores_used(),
                                "kind": "oracle", "sample": f"one head's full table ({el:.1f} s of fp64 numpy), "
                                                           f"extrapolated to {n} heads"}
-    del x, U, lam, omega, mu, signs, coords, D
+    del x, U, lam, w, mu, signs, coords, D
     return out
 
 
@@ -614,12 +614,45 @@ def run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out, cpu_ba
             "gpu_launches": 3 * K}
 
 
-def aux_leg(fn, *a):
-    """The JSON object of a leg measured after the headline, or {"error": ...} if it failed."""
-    try:
-        return fn(*a)
-    except Exception as e:  # the headline line is printed either way
-        return {"error": f"{type(e).__name__}: {e}"[:400]}
+class AuxLegs:
+    """Runs the legs measured after the headline.  A leg that fails is reported in its place as
+    {"error": ...}.  After a device-side failure (a CUDA error, or a library status of
+    COBRA_ECUDA / COBRA_ETIMEOUT, which can leave the context unusable) the remaining GPU legs are
+    not run on that context: each reports {"error": "skipped after ..."} naming the first cause.
+    Every leg ends with a synchronisation and a status check, so a failure is charged to the leg
+    that caused it."""
+
+    def __init__(self, stream):
+        self.stream = stream
+        self.device_error = None
+
+    def _is_device_error(self, e) -> bool:
+        from paper_2609_24298_gb300 import cobra
+
+        if isinstance(e, cobra.CobraError):
+            return e.status in (cobra.COBRA_ECUDA, cobra.COBRA_ETIMEOUT)
+        msg = str(e)
+        return "CUDA" in msg or "cuda" in msg or "device-side" in msg
+
+    def run(self, fn, *a):
+        import torch
+
+        from paper_2609_24298_gb300 import cobra
+
+        if self.device_error:
+            return {"error": f"skipped after {self.device_error}"[:400]}
+        try:
+            res = fn(*a)
+            torch.cuda.synchronize()
+            st = cobra.cobra_check(self.stream)
+            if st != cobra.COBRA_OK:
+                raise cobra.CobraError("cobra_check after " + fn.__name__, st)
+            return res
+        except Exception as e:  # the headline line is printed either way
+            msg = f"{fn.__name__}: {type(e).__name__}: {e}"[:400]
+            if self._is_device_error(e):
+                self.device_error = msg
+            return {"error": msg}
 
 
 def run_cobra(args):
@@ -662,7 +695,9 @@ def run_cobra(args):
         gbs, n, el = oracle_rate(args.cpu_seconds, T, G)
         cpu = {"value": gbs, "unit": "GB/s", "cores": cores_used(), "kind": "oracle",
                "sample": f"{n} (seq, layer, kv-head) decode steps over {T} tokens with K and V at r={SAMPLE_R}, "
-                         f"b={SAMPLE_B} incl. append-compress ({el:.1f} s of fp64 numpy)"}
+                         f"b={SAMPLE_B} incl. append-compress ({el:.1f} s of fp64 numpy); a fixed-allocation sample: at "
+                         "1 bpd every head stores r b = 128 bits per token, the same bytes as the allocated heads, "
+                         "whose (r, b) vary"}
 
     k_bpd = args.k_bpd if args.k_bpd is not None else spec["bpd"]
     v_opts = cobra.alloc_opts(mode=cobra.ALLOC_UNIFORM) if args.v_uniform else None
@@ -807,20 +842,21 @@ def run_cobra(args):
     peak, peak_kind = hbm_peak()
     achieved = bytes_step / (scan_ms * 1e-3) / 1e9
     # the legs below are measured after the headline: a failure in one is reported in its place
+    legs = AuxLegs(stream)
     calibration = None
     if not args.no_calibration and rank == 0:
-        calibration = aux_leg(run_calibration_leg, args, dev, stream, srcs, not args.no_cpu_baseline and world == 1)
+        calibration = legs.run(run_calibration_leg, args, dev, stream, srcs, not args.no_cpu_baseline and world == 1)
     measured = None
     if not args.no_measured and rank == 0:
-        measured = aux_leg(run_measured_leg, args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
+        measured = legs.run(run_measured_leg, args, dev, stream, hp.cals, srcs, not args.no_cpu_baseline and world == 1)
     rope = None
     if not args.no_rope and rank == 0:
-        rope = aux_leg(run_rope_leg, args, dev, stream, hp, wl, desc, ws, info, q, lens, out,
-                       not args.no_cpu_baseline and world == 1)
+        rope = legs.run(run_rope_leg, args, dev, stream, hp, wl, desc, ws, info, q, lens, out,
+                        not args.no_cpu_baseline and world == 1)
     compress = None
     if not args.no_compress:
         del hin, hout
-        compress = aux_leg(run_compress_leg, args, dev, stream, peak)
+        compress = legs.run(run_compress_leg, args, dev, stream, peak)
     traffic = profiled_traffic()
     if rank == 0:
         line = {
