@@ -60,6 +60,9 @@ def parse_args():
     ap.add_argument("--calibration-only", action="store_true", help="only the device calibration leg")
     ap.add_argument("--no-rope", action="store_true", help="skip the RoPE decode leg")
     ap.add_argument("--rope-steps", type=int, default=20, help="timed calls of the RoPE decode leg")
+    ap.add_argument("--no-configs", action="store_true", help="skip the config 1, 3 and 5 decode legs")
+    ap.add_argument("--configs-only", action="store_true", help="only the config 1, 3 and 5 decode legs")
+    ap.add_argument("--config-steps", type=int, default=30, help="timed steps of the config 3 and 5 legs")
     return ap.parse_args()
 
 
@@ -614,6 +617,229 @@ def run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out, cpu_ba
             "gpu_launches": 3 * K}
 
 
+# ---------------------------------------------------------------------------------------
+# the other decode workloads (configs 1, 3 and 5), measured after the headline
+# ---------------------------------------------------------------------------------------
+def allocated_params(cfg: int, layers: int, bpd: float, base=None):
+    """Per-head parameters of a config at `bpd`: calibration (reused from `base` when given:
+    the rate sweep re-allocates the same calibrated heads) and the library's allocation."""
+    from paper_2609_24298_gb300 import cobra, pipeline, synth
+
+    spec = synth.CONFIGS[cfg]
+    if base is None:
+        return pipeline.build_params(cfg, layers, bpd, joint=spec["joint"])
+    hp0, srcs = base
+    w = hp0.alloc["w"]
+    if spec["joint"]:
+        res = cobra.cobra_allocate(w, bpd)
+        r, b = res["r"], res["b"]
+    else:
+        n = len(w) // 2
+        rk, rv = cobra.cobra_allocate(w[:n], bpd), cobra.cobra_allocate(w[n:], bpd)
+        r, b = np.concatenate([rk["r"], rv["r"]]), np.concatenate([rk["b"], rv["b"]])
+    hp = pipeline.fuse_heads(hp0.cals, r, b, [synth.hadamard_signs(*x.key) for x in srcs])
+    hp.cals, hp.alloc = hp0.cals, hp0.alloc
+    return hp, srcs
+
+
+class StepWorkload:
+    """A decode workload on the device: the cache filled by cobra_compress with T - 1 tokens per
+    sequence, the plan, and the inputs of one decode step (append of the new K and V token at
+    position T - 1, query projection, scan, combine; cobra_decode_step)."""
+
+    def __init__(self, dev, cfg: int, layers: int, hp, srcs, lens, paged: bool, seed: int):
+        import torch
+
+        from paper_2609_24298_gb300 import cobra, pipeline, synth
+
+        spec = synth.CONFIGS[cfg]
+        H = spec["kv_heads"]
+        G = spec["q_heads"] // H
+        L, S = layers, len(lens)
+        lens = np.asarray(lens, np.int64)
+        rows = int(-(-lens.max() // 128))
+        wl = pipeline.Workload(cfg=cfg, layers=L, kv=H, group=G, seqs=S, tokens=lens - 1, bpd=0.0, joint=False)
+        if paged:
+            pps = -(-rows // 2)
+            wl.pages_per_seq = pps
+            wl.page_table = torch.tensor(synth.shuffled_pages(cfg, S * pps), dtype=torch.int32, device=dev)
+            n_slots = 2 * S * pps
+        else:
+            wl.rows_per_seq = rows
+            n_slots = S * rows
+        wl.dev = pipeline.DeviceParams(hp, n_slots, device=dev)
+        pipeline.fill_cache(wl, srcs, device=dev)
+        wl.tokens = lens
+        self.desc, self.ws, self.info = pipeline.decode_setup(wl, device=dev)
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(seed)
+        self.xk = torch.randn((L, S, H, 128), generator=gen, device=dev).to(torch.bfloat16)
+        self.xv = torch.randn((L, S, H, 128), generator=gen, device=dev).to(torch.bfloat16)
+        self.q = torch.randn((L, S, H * G, 128), generator=gen, device=dev).to(torch.bfloat16)
+        self.out = torch.empty((L, S, H * G, 128), dtype=torch.float32, device=dev)
+        self.pos = torch.tensor(lens - 1, dtype=torch.int32, device=dev)
+        self.lens = torch.tensor(lens, dtype=torch.int32, device=dev)
+        self.adesc = [cobra.compress_desc(head0=side * L * H, layer_stride=H, n_layers=L, n_kv_heads=H, side=side,
+                                          n_seqs=S, rows_per_seq=wl.rows_per_seq, pages_per_seq=wl.pages_per_seq,
+                                          x_stride_layer=S * H * 128, x_stride_seq=H * 128, x_stride_tok=0,
+                                          x_stride_head=128) for side in (0, 1)]
+        self.wl, self.hp, self.G = wl, hp, G
+        self.bytes = pipeline.packed_bytes_read(wl)
+
+    def step(self, stream):
+        from paper_2609_24298_gb300 import cobra
+
+        wl = self.wl
+        cobra.cobra_decode_step(wl.dev.block, self.desc, self.info, self.adesc[0], self.adesc[1], self.xk, self.xv,
+                                self.pos, self.q, wl.dev.cache, self.lens, wl.page_table, self.out, self.ws,
+                                self.ws.numel(), stream)
+
+    def scan(self, stream):
+        from paper_2609_24298_gb300 import cobra
+
+        wl = self.wl
+        cobra.cobra_decode_scan(wl.dev.block, self.desc, self.info, wl.dev.cache, self.lens, wl.page_table, self.ws,
+                                self.ws.numel(), stream)
+
+    def timed(self, stream, steps: int, warmup: int):
+        """(ms per step, ms per scan): K steps with events at the two ends only, then the scan
+        alone between events (the q~ blocks of the last step stay in the workspace)."""
+        import torch
+
+        from paper_2609_24298_gb300 import cobra
+
+        for _ in range(warmup):
+            self.step(stream)
+        torch.cuda.synchronize()
+        if cobra.cobra_check(stream) != cobra.COBRA_OK:
+            raise RuntimeError("device status after warm-up")
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev[0].record(stream)
+        for _ in range(steps):
+            self.step(stream)
+        ev[1].record(stream)
+        ev[2].record(stream)
+        for _ in range(steps):
+            self.scan(stream)
+        ev[3].record(stream)
+        torch.cuda.synchronize()
+        if cobra.cobra_check(stream) != cobra.COBRA_OK:
+            raise RuntimeError("device status after the timed steps")
+        return ev[0].elapsed_time(ev[1]) / steps, ev[2].elapsed_time(ev[3]) / steps
+
+    def release(self):
+        del self.wl, self.ws, self.xk, self.xv, self.q, self.out
+
+
+def oracle_group_rate(hp, srcs, cfg: int, layers: int, T: int, G: int, seconds: float):
+    """The fp64 oracle's decode of one (layer 0, kv head 0) group of a leg's workload over T
+    tokens, with that group's allocated (r, b) (compressing its context is setup, not timed),
+    repeated for about `seconds`.  Returns (GB/s of packed codes, groups done, seconds)."""
+    from oracle import attention as oatt
+    from oracle import compress as ocomp
+    from paper_2609_24298_gb300 import synth
+
+    spec = synth.CONFIGS[cfg]
+    H = spec["kv_heads"]
+    n = layers * H
+    ps, codes, nbytes = [], [], 0
+    for idx in (0, n):  # K and V head of (layer 0, kv head 0)
+        r, b = int(hp.r[idx]), int(hp.b[idx]) if hp.r[idx] else 1
+        p = {"r": r, "b": b, "W": np.asarray(hp.W[idx], np.float32), "delta": np.float32(hp.delta[idx]),
+             "mu": np.asarray(hp.mu[idx], np.float32)}
+        if r:
+            _, c = ocomp.compress(srcs[idx].tokens(T), p["W"], p["mu"], p["delta"], b)
+        else:
+            c = np.zeros((T, 0), np.int64)
+        ps.append(p)
+        codes.append(c)
+        nbytes += ((T * r * (b if r else 0) + 7) // 8 + 15) // 16 * 16
+    q = synth.decode_queries(cfg, 0, 0, 1, G)[0].astype(np.float64)
+    done, t0 = 0, time.perf_counter()
+    while True:
+        oatt.decode(q, codes[0], codes[1], ps[0], ps[1])
+        done += 1
+        el = time.perf_counter() - t0
+        if el >= seconds and done >= 1:
+            break
+    return nbytes * done / el / 1e9, done, el
+
+
+def workload_leg(args, dev, stream, cfg: int, bpd: float, lens, paged: bool, steps: int, cpu_baseline: bool,
+                 base=None, label: str = ""):
+    """One decode workload measured like the headline (cobra_decode_step, events at the ends of
+    the timed steps; the scan alone for its roofline).  Returns (JSON object, (hp, srcs))."""
+    from paper_2609_24298_gb300 import synth
+
+    spec = synth.CONFIGS[cfg]
+    H = spec["kv_heads"]
+    G = spec["q_heads"] // H
+    L = spec["layers"]
+    hp, srcs = allocated_params(cfg, L, bpd, base)
+    wlk = StepWorkload(dev, cfg, L, hp, srcs, lens, paged, seed=cfg * 7919 + int(bpd * 8))
+    ms, scan_ms = wlk.timed(stream, steps, args.warmup)
+    peak, kind = hbm_peak()
+    achieved = wlk.bytes / (scan_ms * 1e-3) / 1e9
+    out = {"workload": label, "bpd": bpd, "value": wlk.bytes / (ms * 1e-3) / 1e9, "unit": "GB/s",
+           "ms_per_step": ms, "steps": steps, "packed_bytes_per_step": wlk.bytes,
+           "roofline": {"bound": "hbm", "kernel": "decode_kernel (rank-space scan)", "achieved": achieved,
+                        "peak": peak, "peak_kind": kind, "unit": "GB/s", "frac": achieved / peak,
+                        "scan_ms": scan_ms},
+           "gpu_launches": 4 * (steps + args.warmup) + steps}
+    wlk.release()
+    if cpu_baseline:
+        gbs, n, el = oracle_group_rate(hp, srcs, cfg, L, int(np.asarray(lens)[0]), G, args.cpu_seconds / 3)
+        out["cpu_baseline"] = {"value": gbs, "unit": "GB/s", "cores": cores_used(), "kind": "oracle",
+                               "sample": f"{n} decode(s) of one (layer 0, kv head 0) group over "
+                                         f"{int(np.asarray(lens)[0])} tokens with its allocated (r_K, b_K) = "
+                                         f"({int(hp.r[0])}, {int(hp.b[0])}), (r_V, b_V) = "
+                                         f"({int(hp.r[L * H])}, {int(hp.b[L * H])}) ({el:.1f} s of fp64 numpy)"}
+    return out, (hp, srcs)
+
+
+def run_config3_leg(args, dev, stream, cpu_baseline: bool):
+    """Llama-3-70B-shaped joint K+V at 0.5 bpd: 80 layers x 8 kv heads, GQA 8, one 131072-token
+    sequence; the step appends the new token and decodes over all layers."""
+    from paper_2609_24298_gb300 import synth
+
+    spec = synth.CONFIGS[3]
+    out, _ = workload_leg(args, dev, stream, 3, spec["bpd"], [spec["tokens"]], False, args.config_steps,
+                          cpu_baseline, label="llama3-70b-shaped decode step: 80 layers x 8 kv heads (GQA 8) x 1 "
+                                              "sequence x 131072 tokens, K and V allocated jointly at 0.5 bpd")
+    return out
+
+
+def run_config5_leg(args, dev, stream, cpu_baseline: bool):
+    """Ragged paged rate sweep: 32 layers x 8 kv heads x 32 sequences of lengths uniform in
+    [1024, 65536] in 256-token pages (shuffled), every bpd point re-allocated."""
+    from paper_2609_24298_gb300 import synth
+
+    spec = synth.CONFIGS[5]
+    lens = synth.ragged_lengths(5, spec["seqs"], *spec["tokens"])
+    points, base = [], None
+    for i, bpd in enumerate(spec["bpd"]):
+        o, base = workload_leg(args, dev, stream, 5, bpd, lens, True, args.config_steps, cpu_baseline and i == 1,
+                               base=base, label=f"ragged paged sweep point: 32 layers x 8 kv heads x 32 sequences "
+                                                f"(lengths in [1024, 65536], sum {int(lens.sum())}), 256-token "
+                                                f"pages, K and V at {bpd} bpd")
+        points.append(o)
+    return {"workload": "ragged paged rate sweep (configs[4] shape)", "points": points}
+
+
+def run_config1_leg(args, dev, stream, cpu_baseline: bool):
+    """The tiny single-layer case: 8 kv heads, GQA 4, one 2048-token sequence at 2 bpd; the
+    decode step's latency."""
+    from paper_2609_24298_gb300 import synth
+
+    spec = synth.CONFIGS[1]
+    out, _ = workload_leg(args, dev, stream, 1, spec["bpd"], [spec["tokens"]], False, 200, cpu_baseline,
+                          label="tiny decode step: 1 layer x 8 kv heads (GQA 4) x 1 sequence x 2048 tokens, "
+                                "K and V at 2 bpd")
+    out["latency_us"] = out["ms_per_step"] * 1e3
+    out["note"] = "latency-bound: the packed bytes (1 MB) fit L2 and the step is four short launches"
+    return out
+
+
 class AuxLegs:
     """Runs the legs measured after the headline.  A leg that fails is reported in its place as
     {"error": ...}.  After a device-side failure (a CUDA error, or a library status of
@@ -682,6 +908,13 @@ def run_cobra(args):
         srcs = [synth.HeadSource(CFG, l, h, side, spec["alpha"]) for side in (0, 1) for l in range(L) for h in range(H)]
         print(json.dumps(run_calibration_leg(args, dev, torch.cuda.current_stream(), srcs,
                                              not args.no_cpu_baseline)), flush=True)
+        return
+    if args.configs_only:
+        legs = AuxLegs(torch.cuda.current_stream())
+        st, cb = torch.cuda.current_stream(), not args.no_cpu_baseline
+        print(json.dumps({"config1_tiny": legs.run(run_config1_leg, args, dev, st, cb),
+                          "config3_llama3_70b_joint": legs.run(run_config3_leg, args, dev, st, cb),
+                          "config5_ragged_sweep": legs.run(run_config5_leg, args, dev, st, cb)}), flush=True)
         return
     if args.measured_only:
         hp, srcs = pipeline.build_params(CFG, L, spec["bpd"], joint=False)
@@ -853,6 +1086,12 @@ def run_cobra(args):
     if not args.no_rope and rank == 0:
         rope = legs.run(run_rope_leg, args, dev, stream, hp, wl, desc, ws, info, q, lens, out,
                         not args.no_cpu_baseline and world == 1)
+    configs = None
+    if not args.no_configs and rank == 0:
+        cb = not args.no_cpu_baseline and world == 1
+        configs = {"config1_tiny": legs.run(run_config1_leg, args, dev, stream, cb),
+                   "config3_llama3_70b_joint": legs.run(run_config3_leg, args, dev, stream, cb),
+                   "config5_ragged_sweep": legs.run(run_config5_leg, args, dev, stream, cb)}
     compress = None
     if not args.no_compress:
         del hin, hout
@@ -870,6 +1109,7 @@ def run_cobra(args):
                          "traffic": traffic, "scan_ms": scan_ms,
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
             "compress": compress,
+            "other_decode_configs": configs,
             "rope": rope,
             "measured": measured,
             "calibration": calibration,
