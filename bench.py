@@ -61,7 +61,7 @@ def parse_args():
     ap.add_argument("--no-rope", action="store_true", help="skip the RoPE decode leg")
     ap.add_argument("--rope-steps", type=int, default=20, help="timed calls of the RoPE decode leg")
     ap.add_argument("--no-configs", action="store_true", help="skip the config 1, 3 and 5 decode legs")
-    ap.add_argument("--configs-only", action="store_true", help="only the config 1, 3 and 5 decode legs")
+    ap.add_argument("--configs-only", default=None, help="only these of the config 1, 3, 5 decode legs, e.g. 1,3,5")
     ap.add_argument("--config-steps", type=int, default=30, help="timed steps of the config 3 and 5 legs")
     return ap.parse_args()
 
@@ -912,9 +912,11 @@ def run_cobra(args):
     if args.configs_only:
         legs = AuxLegs(torch.cuda.current_stream())
         st, cb = torch.cuda.current_stream(), not args.no_cpu_baseline
-        print(json.dumps({"config1_tiny": legs.run(run_config1_leg, args, dev, st, cb),
-                          "config3_llama3_70b_joint": legs.run(run_config3_leg, args, dev, st, cb),
-                          "config5_ragged_sweep": legs.run(run_config5_leg, args, dev, st, cb)}), flush=True)
+        todo = {int(x) for x in args.configs_only.split(",")}
+        fns = {1: ("config1_tiny", run_config1_leg), 3: ("config3_llama3_70b_joint", run_config3_leg),
+               5: ("config5_ragged_sweep", run_config5_leg)}
+        print(json.dumps({name: legs.run(fn, args, dev, st, cb) for c, (name, fn) in fns.items() if c in todo}),
+              flush=True)
         return
     if args.measured_only:
         hp, srcs = pipeline.build_params(CFG, L, spec["bpd"], joint=False)

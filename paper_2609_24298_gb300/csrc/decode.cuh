@@ -590,7 +590,17 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
         default: scan_item<G, 0, 0>(a, w, item); break;
       }
     } else {
-      scan_item<G, 0, 0>(a, w, item);
+      // G = 8 (low rates: the 1- and 2-bit pairs carry nearly all of the cache)
+      const WsGroup gr = groups[items[item].group];
+      const HeadEntry hk = heads[gr.k_head], hv = heads[gr.v_head];
+      const int key = (hk.r > 0 ? hk.b : 0) * 16 + (hv.r > 0 ? hv.b : 0);
+      switch (key) {
+        case 0x11: scan_item<G, 1, 1>(a, w, item); break;
+        case 0x12: scan_item<G, 1, 2>(a, w, item); break;
+        case 0x21: scan_item<G, 2, 1>(a, w, item); break;
+        case 0x22: scan_item<G, 2, 2>(a, w, item); break;
+        default: scan_item<G, 0, 0>(a, w, item); break;
+      }
     }
   }
   if (w.failed) {
