@@ -242,3 +242,56 @@ def test_kv_split_with_uniform_v(k_bpd, v_bpd):
     params = [ocal.head_params(c, int(rr), int(bb) if rr else 1, synth.hadamard_signs(*s.key))
               for c, s, rr, bb in zip(cals, srcs, r, b)]
     run_workload(2, 4, params, srcs, [32768] * 8, [(0, 0, 0), (1, 5, 3), (3, 7, 7)])
+
+
+def test_prefill_compress_full_size():
+    """The prefill workload compressed in the benchmark's launch geometry: 32 layers x 8 kv heads
+    x batch 64 x 4096 tokens of bf16 K and V at 4 bpd (about 34 GB of input), one cobra_compress
+    launch per side over all layers (the grid of (layer, head, tile chunk) CTAs the benchmark
+    times).  Sampled (layer, kv head, side, sequence, token range) slices: codes equal the
+    oracle's, or differ by one within 1e-4 of a cell boundary, and re-packing the kernel's codes
+    with the oracle's packer reproduces the rows bit for bit (Table alg:kvrobin step 7)."""
+    spec = synth.CONFIGS[4]
+    L, H, S, T = spec["layers"], spec["kv_heads"], spec["seqs"], spec["tokens"]
+    cals, srcs = oracle_calibrations(4, L)
+    params = oracle_allocated_params(cals, srcs, spec["bpd"])
+    hp = oracle_head_params(params)
+    rows = T // 128
+    dp = pipeline.DeviceParams(hp, S * rows, device=DEV)
+    # (layer, kv head, side, seq, first token, tokens)
+    samples = [(0, 0, 0, 0, 0, 384), (0, 7, 1, 63, 3712, 384), (13, 3, 0, 31, 1000, 700),
+               (31, 5, 1, 17, 0, 4096), (31, 0, 0, 40, 2048, 256), (22, 6, 1, 5, 128, 130)]
+    xs = {}
+    for side in (0, 1):
+        x = torch.empty((L, S, T, H, D), dtype=torch.bfloat16, device=DEV)
+        for l in range(L):
+            x[l] = pipeline.device_tokens([srcs[side * L * H + l * H + h] for h in range(H)], S, T,
+                                          seed=4 * 1000003 + 2 * l + side, device=DEV)
+        desc = cobra.compress_desc(head0=side * L * H, layer_stride=H, n_layers=L, n_kv_heads=H, side=side, n_seqs=S,
+                                   rows_per_seq=rows, x_stride_layer=S * T * H * D, x_stride_seq=T * H * D,
+                                   x_stride_tok=H * D, x_stride_head=D)
+        cobra.cobra_compress(dp.block, desc, x, 0, T, dp.cache)
+        for (l, h, sd, q, t0, n) in samples:
+            if sd == side:
+                xs[(l, h, q, t0, n)] = x[l, q, t0:t0 + n, h].float().cpu().numpy()
+        del x
+    torch.cuda.synchronize()
+    assert cobra.cobra_check() == cobra.COBRA_OK
+    for (l, h, side, q, t0, n) in samples:
+        idx = side * L * H + l * H + h
+        p = params[idx]
+        r, b = p["r"], p["b"]
+        if r == 0:
+            continue
+        rb = olay.row_bytes(r, b)
+        base = int(dp.offsets[idx]) + q * rows * rb
+        host_rows = dp.cache[base:base + rows * rb].cpu().numpy()
+        got_all = read_head_codes(host_rows, 0, side, r, b, T, seq=0, rows_per_seq=rows)
+        x = xs[(l, h, q, t0, n)]
+        u, want = ocomp.compress(x, p["W"], p["mu"], p["delta"], b)
+        got = got_all[t0:t0 + n]
+        assert codes_ok(got, u, want), (l, h, side, q, np.argwhere(got != want)[:5])
+        # the rows holding the slice, re-packed from the kernel's own codes, are its bytes
+        rep = olay.pack_tokens(got_all, side, b)
+        for row in range(t0 // 128, -(-(t0 + n) // 128)):
+            assert np.array_equal(rep[row], host_rows[row * rb:(row + 1) * rb]), (l, h, side, q, row)
