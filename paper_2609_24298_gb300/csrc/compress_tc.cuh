@@ -4,7 +4,7 @@
 //
 // One CTA per (layer, kv head) and chunk of 128-token tiles, 6 warps:
 //   warp 0    TMA producer: each tile X [128 tokens x 128 dims] bf16 arrives as two 64-dim
-//             boxes with 128-byte swizzle into a 3-stage shared-memory ring.
+//             boxes with 128-byte swizzle into a shared-memory ring of 5 (b <= 5) or 4 stages.
 //   warp 1    allocates TMEM; one thread issues tcgen05.mma computing the transposed
 //             projection Y^T = W X^T (M = 128 channels, rows past r zero; N = 128 tokens;
 //             K = 16 per instruction; bf16 inputs, fp32 accumulation in TMEM).  The head's
@@ -33,11 +33,14 @@ namespace cobra {
 constexpr int kTcThreads = 192;
 constexpr uint64_t kTcWaitNs = 2000000000ull;  // 2 s
 constexpr int kTcEpiWarp0 = 2;
-constexpr int kTcStages = 3;               // X ring
 constexpr int kTcTmemCols = 256;           // two accumulators of 128 columns (tokens)
 constexpr int kTcXStageBytes = 2 * 16384;  // two 64-dim swizzle atoms of 128 rows
-constexpr int kTcWBytes = 3 * 2 * 128 * 128;
-constexpr int kTcSmemBytes = 1024 + kTcWBytes + kTcStages * kTcXStageBytes + 256;
+constexpr int kTcSplitBytes = 2 * 16384;   // one bf16 term of the basis, same layout
+// The basis terms and the X ring share one region of seven 32 KB slots: 2 terms + 5 stages
+// (b <= 5) or 3 terms + 4 stages (b >= 6).
+constexpr int kTcSlots = 7;
+constexpr int kTcStagesMax = 5;
+constexpr int kTcSmemBytes = 1024 + kTcSlots * kTcXStageBytes + 256;
 
 struct TcArgs {
   const unsigned char* block;
@@ -93,6 +96,18 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&v)[32]) {
       : "memory");
 }
 __device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// The same wait, with v (the destination of the load in flight) passed through it, so that no
+// use of v can be scheduled ahead of the wait.
+__device__ __forceinline__ void tc_wait_ld(uint32_t (&v)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
+                 "+r"(v[8]), "+r"(v[9]), "+r"(v[10]), "+r"(v[11]), "+r"(v[12]), "+r"(v[13]), "+r"(v[14]), "+r"(v[15]),
+                 "+r"(v[16]), "+r"(v[17]), "+r"(v[18]), "+r"(v[19]), "+r"(v[20]), "+r"(v[21]), "+r"(v[22]),
+                 "+r"(v[23]), "+r"(v[24]), "+r"(v[25]), "+r"(v[26]), "+r"(v[27]), "+r"(v[28]), "+r"(v[29]),
+                 "+r"(v[30]), "+r"(v[31])
+               :
+               : "memory");
+}
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
@@ -114,9 +129,32 @@ __device__ __forceinline__ uint32_t umma_idesc_bf16(int M, int N) {
 
 // Epilogue state of one thread (one channel).
 struct TcEpi {
-  float inv_delta, cterm;  // u = y inv_delta + cterm, cterm = 2^{b-1} - (W^T mu)_i inv_delta
-  int cmax;
+  // u = y inv_delta + cterm with cterm = 2^{b-1} - (W^T mu)_i inv_delta, both scaled by 2^-b
+  // (exact): s = u 2^-b
+  float inv_s, cterm_s;
+  uint32_t top;  // bit pattern of kTcMagic + 2^b - 1
 };
+
+// Rounding down without a float-to-integer conversion: for s in [0, 1], the fp32 sum
+// kTcMagic + s 2^b rounded toward -inf is kTcMagic + floor(s 2^b) (the spacing of fp32 values
+// in [2^23, 2^24) is 1), so its bit pattern is kTcMagicBits + floor(s 2^b).
+constexpr float kTcMagic = 12582912.0f;  // 1.5 * 2^23
+constexpr uint32_t kTcMagicBits = 0x4B400000u;
+
+// Each code enters its sub-stream word as (kTcMagicBits + code) << off (and, for a code that
+// straddles two words, (kTcMagicBits + code) >> (32 - off) in the next one).  The constant
+// parts are disjoint from the code bits, so they add up to a fixed sum per word; starting the
+// word at minus that sum leaves exactly the codes once all 16 of the sub-stream's codes are in.
+template <int B>
+__host__ __device__ constexpr uint32_t tc_word_init(int k) {
+  uint32_t acc = 0u;
+  for (int rho = 0; rho < 16; ++rho) {
+    const int pos = rho * B, kk = pos >> 5, off = pos & 31;
+    if (kk == k) acc += kTcMagicBits << off;
+    if (off + B > 32 && kk + 1 == k) acc += kTcMagicBits >> (32 - off);
+  }
+  return 0u - acc;
+}
 
 // Codes of the 32 tokens 32 c .. 32 c + 31 of this thread's channel into its sub-streams:
 // token t -> sub-stream t % 8, bits [(t / 8) B, (t / 8) B + B).
@@ -125,11 +163,13 @@ __device__ __forceinline__ void tc_codes32(const uint32_t (&v)[32], const TcEpi&
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
     const int t = 32 * C + j, sig = t & 7, pos = (t >> 3) * B;
-    int c = __float2int_rd(fmaf(__uint_as_float(v[j]), e.inv_delta, e.cterm));
-    c = min(max(c, 0), e.cmax);
+    // s = clamp(u 2^-b, 0, 1) (NaN -> 0), then kTcMagic + floor(s 2^b), its top clamped at
+    // code 2^b - 1: the bits are kTcMagicBits + clamp(floor(u), 0, 2^b - 1)
+    const float s = __saturatef(fmaf(__uint_as_float(v[j]), e.inv_s, e.cterm_s));
+    const uint32_t c = min(__float_as_uint(__fmaf_rd(s, (float)(1 << B), kTcMagic)), e.top);
     const int k = pos >> 5, off = pos & 31;
-    sub[sig][k] |= (uint32_t)c << off;
-    if (off + B > 32) sub[sig][k + 1] |= (uint32_t)c >> (32 - off);
+    sub[sig][k] += c << off;
+    if (off + B > 32) sub[sig][k + 1] += c >> (32 - off);
   }
 }
 
@@ -192,22 +232,23 @@ __device__ __forceinline__ void tc_epilogue(const TcArgs& a, const HeadEntry& he
 #pragma unroll
     for (int s = 0; s < 8; ++s)
 #pragma unroll
-      for (int k = 0; k < NW; ++k) sub[s][k] = 0u;
+      for (int k = 0; k < NW; ++k) sub[s][k] = tc_word_init<B>(k);
     const uint32_t tb = tmem_q + (uint32_t)(acc * 128);
     {
-      uint32_t v[32];
-      tc_ld32(tb + 0, v);
-      tc_wait_ld();
-      tc_codes32<B, 0>(v, e, sub);
-      tc_ld32(tb + 32, v);
-      tc_wait_ld();
-      tc_codes32<B, 1>(v, e, sub);
-      tc_ld32(tb + 64, v);
-      tc_wait_ld();
-      tc_codes32<B, 2>(v, e, sub);
-      tc_ld32(tb + 96, v);
-      tc_wait_ld();
-      tc_codes32<B, 3>(v, e, sub);
+      // each load of 32 columns is in flight while the previous 32 are quantised
+      uint32_t v0[32], v1[32];
+      tc_ld32(tb + 0, v0);
+      tc_wait_ld(v0);
+      tc_ld32(tb + 32, v1);
+      tc_codes32<B, 0>(v0, e, sub);
+      tc_wait_ld(v1);
+      tc_ld32(tb + 64, v0);
+      tc_codes32<B, 1>(v1, e, sub);
+      tc_wait_ld(v0);
+      tc_ld32(tb + 96, v1);
+      tc_codes32<B, 2>(v0, e, sub);
+      tc_wait_ld(v1);
+      tc_codes32<B, 3>(v1, e, sub);
     }
     // the accumulator can take the next tile's MMAs
     tc_fence_before();
@@ -246,11 +287,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);  // 1024-aligned for the swizzle
-  uint8_t* wsm = base;                                           // [split][atom][128 channels][128 B]
-  uint8_t* xsm = wsm + kTcWBytes;                                // [stage][atom][128 tokens][128 B]
-  // x_full[kTcStages] x_empty[kTcStages] acc_full[2] acc_empty[2] done
-  uint64_t* bars = reinterpret_cast<uint64_t*>(xsm + kTcStages * kTcXStageBytes);
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * kTcStages + 5);
+  uint8_t* wsm = base;  // [split][atom][128 channels][128 B], then the X ring
+  // x_full[kTcStagesMax] x_empty[kTcStagesMax] acc_full[2] acc_empty[2] done
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + kTcSlots * kTcXStageBytes);
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * kTcStagesMax + 5);
   int* counters = reinterpret_cast<int*>(tmem_holder + 1);  // [0] tiles issued by TMA, [1] consumed by MMA, [2] fail
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -262,16 +302,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int ntiles = a.n_seqs * nrows;
   if (r == 0 || chunk >= ntiles) return;
   const int my_tiles = (ntiles - chunk + a.chunks - 1) / a.chunks;
-  const int nsplit = b >= 6 ? 3 : 2;
+  const int nsplit = b >= 6 ? 3 : 2, nstage = kTcSlots - nsplit;
+  uint8_t* xsm = wsm + nsplit * kTcSplitBytes;  // [stage][atom][128 tokens][128 B]
   const float* pool = param_pool(a.block);
   const float* W = pool + he.w_off;
   const uint32_t bar0 = smem_addr(bars);
   auto bar = [&](int i) { return bar0 + 8u * i; };
-  const int XF = 0, XE = kTcStages, AF = 2 * kTcStages, AE = 2 * kTcStages + 2, DONE = 2 * kTcStages + 4;
+  const int XF = 0, XE = kTcStagesMax, AF = 2 * kTcStagesMax, AE = AF + 2, DONE = AF + 4;
 
   // ---- setup: barriers, TMEM, split basis ----
   if (tid == 0) {
-    for (int i = 0; i < kTcStages; ++i) {
+    for (int i = 0; i < nstage; ++i) {
       mbar_init(bar(XF + i), 1);  // producer arrive + TMA bytes
       mbar_init(bar(XE + i), 1);  // MMA commit
     }
@@ -320,7 +361,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             rem[2 * e2 + 1] -= p1;
             packed[e2] = pack_bf16(p0, p1);
           }
-          uint8_t* rowp = wsm + (size_t)sp * 2 * 128 * 128 + (size_t)atom * 128 * 128 + (size_t)n * 128;
+          uint8_t* rowp = wsm + (size_t)sp * kTcSplitBytes + (size_t)atom * 128 * 128 + (size_t)n * 128;
           *reinterpret_cast<uint4*>(rowp + ((c ^ (n & 7)) << 4)) =
               make_uint4(packed[0], packed[1], packed[2], packed[3]);
         }
@@ -339,7 +380,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       int issued = 0;
       for (int i = 0; i < my_tiles; ++i) {
-        const int st = i % kTcStages, ph = (i / kTcStages) & 1;
+        const int st = i % nstage, ph = (i / nstage) & 1;
         if (!mbar_wait_bounded(bar(XE + st), ph ^ 1, kTcWaitNs)) {
           atomicOr(&g_status, 1u);
           counters[2] = 1;
@@ -369,8 +410,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const uint32_t wbase = smem_addr(wsm), xbase = smem_addr(xsm);
       int consumed = 0;
       for (int i = 0; i < my_tiles; ++i) {
-        const int st = i % kTcStages, acc = i & 1;
-        if (!mbar_wait_bounded(bar(XF + st), (i / kTcStages) & 1, kTcWaitNs) ||
+        const int st = i % nstage, acc = i & 1;
+        if (!mbar_wait_bounded(bar(XF + st), (i / nstage) & 1, kTcWaitNs) ||
             !mbar_wait_bounded(bar(AE + acc), ((i >> 1) & 1) ^ 1, kTcWaitNs)) {
           atomicOr(&g_status, 1u);
           counters[2] = 1;
@@ -384,7 +425,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
             const uint32_t koff = (uint32_t)((kk >> 2) * 16384 + (kk & 3) * 32);
-            tc_mma_bf16(d, umma_desc_sw128(wbase + sp * 2 * 16384 + koff),
+            tc_mma_bf16(d, umma_desc_sw128(wbase + sp * kTcSplitBytes + koff),
                         umma_desc_sw128(xbase + st * kTcXStageBytes + koff), idesc, (sp > 0 || kk > 0) ? 1u : 0u);
           }
         tc_commit(bar(XE + st));   // X stage free once these MMAs completed
@@ -398,9 +439,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // ---------------- epilogue (warps 2..5): one channel per thread ----------------
     const int ch = 32 * (warp & 3) + lane;
     TcEpi e;
-    e.inv_delta = he.inv_delta;
-    e.cterm = (float)(1 << (b - 1)) - (ch < r ? pool[he.wmu_off + ch] : 0.f) * he.inv_delta;
-    e.cmax = (1 << b) - 1;
+    const float scale = 1.0f / (float)(1 << b);  // a power of two: the scaled values are exact
+    e.inv_s = he.inv_delta * scale;
+    e.cterm_s = ((float)(1 << (b - 1)) - (ch < r ? pool[he.wmu_off + ch] : 0.f) * he.inv_delta) * scale;
+    e.top = kTcMagicBits + (1u << b) - 1u;
     const uint32_t tq = tmem + ((uint32_t)(32 * (warp & 3)) << 16);  // this warp's TMEM lane quarter
     switch (b) {
       case 1: tc_epilogue<1>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
@@ -417,7 +459,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   if (tid == 0) {
     for (int i = counters[1]; i < counters[0]; ++i)
-      if (!mbar_wait_bounded(bar(XF + i % kTcStages), (i / kTcStages) & 1, kTcWaitNs)) break;
+      if (!mbar_wait_bounded(bar(XF + i % nstage), (i / nstage) & 1, kTcWaitNs)) break;
   }
   tc_fence_before();
   __syncthreads();
