@@ -4,15 +4,16 @@
 //
 // One CTA per (layer, kv head) and chunk of 128-token tiles, 6 warps:
 //   warp 0    TMA producer: each tile X [128 tokens x 128 dims] bf16 arrives as two 64-dim
-//             boxes with 128-byte swizzle into a shared-memory ring of 5 (b <= 5) or 4 stages.
+//             boxes with 128-byte swizzle into a 7-stage shared-memory ring.
 //   warp 1    allocates TMEM; one thread issues tcgen05.mma computing the transposed
 //             projection Y^T = W X^T (M = 128 channels, rows past r zero; N = 128 tokens;
 //             K = 16 per instruction; bf16 inputs, fp32 accumulation in TMEM).  The head's
 //             fp32 basis is split once per CTA into 2 (b <= 5) or 3 (b >= 6) bf16 terms
-//             W = W0 + W1 (+ W2) held in shared memory in the same swizzled K-major layout as
-//             X, so W0 X^T + W1 X^T (+ W2 X^T) reproduces the fp32 projection.  Two TMEM
-//             accumulators alternate between tiles.
-//   warps 2-5 epilogue: a thread owns one channel (its TMEM lane) and reads the 128 token
+//             W = W0 + W1 (+ W2), so W0 X^T + W1 X^T (+ W2 X^T) reproduces the fp32
+//             projection.  The terms are the MMAs' A operand in TMEM, so the tensor cores read
+//             only X from shared memory.  Two TMEM accumulators alternate between tiles.
+//   warps 2-5 write the basis terms into TMEM (a thread per channel), then run the
+//             epilogue: a thread owns one channel (its TMEM lane) and reads the 128 token
 //             values of its row of Y^T.  Token t's code goes to bits [(t/8) b, (t/8) b + b)
 //             of the channel's sub-stream t % 8, which is exactly where format v1 keeps it
 //             (K rows: piece t % 8, code rho = t / 8, half = channel parity; V rows: piece
@@ -33,14 +34,12 @@ namespace cobra {
 constexpr int kTcThreads = 192;
 constexpr uint64_t kTcWaitNs = 2000000000ull;  // 2 s
 constexpr int kTcEpiWarp0 = 2;
-constexpr int kTcTmemCols = 256;           // two accumulators of 128 columns (tokens)
+// TMEM: two accumulators of 128 columns (tokens), then the basis terms (64 columns each)
+constexpr int kTcTmemCols = 512;
+constexpr int kTcWCol = 256;
 constexpr int kTcXStageBytes = 2 * 16384;  // two 64-dim swizzle atoms of 128 rows
-constexpr int kTcSplitBytes = 2 * 16384;   // one bf16 term of the basis, same layout
-// The basis terms and the X ring share one region of seven 32 KB slots: 2 terms + 5 stages
-// (b <= 5) or 3 terms + 4 stages (b >= 6).
-constexpr int kTcSlots = 7;
-constexpr int kTcStagesMax = 5;
-constexpr int kTcSmemBytes = 1024 + kTcSlots * kTcXStageBytes + 256;
+constexpr int kTcStages = 7;               // X ring
+constexpr int kTcSmemBytes = 1024 + kTcStages * kTcXStageBytes + 256;
 
 struct TcArgs {
   const unsigned char* block;
@@ -75,12 +74,14 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
 }
-__device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                            uint32_t accumulate) {
+// D (+)= A B^T, kind::f16 with bf16 inputs: A [M x K] in TMEM (lane = row m, 32-bit column c =
+// elements 2c, 2c + 1 of the row, the lower in the low half), B [N x K] K-major in shared memory.
+__device__ __forceinline__ void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
   asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(
           d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 // 32 consecutive TMEM columns of the warp's 32 lanes: v[j] = column (taddr + j) of this lane
@@ -96,6 +97,16 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&v)[32]) {
       : "memory");
 }
 __device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// 16 consecutive TMEM columns of the warp's 32 lanes: column (taddr + j) of this lane = v[j]
+__device__ __forceinline__ void tc_st32x16(uint32_t taddr, const uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+      "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
+}
+__device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 // The same wait, with v (the destination of the load in flight) passed through it, so that no
 // use of v can be scheduled ahead of the wait.
 __device__ __forceinline__ void tc_wait_ld(uint32_t (&v)[32]) {
@@ -286,11 +297,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     compress_tc_kernel(const __grid_constant__ CUtensorMap xmap, TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
-  uint8_t* base = smem_raw + (((raw + 1023u) & ~1023u) - raw);  // 1024-aligned for the swizzle
-  uint8_t* wsm = base;  // [split][atom][128 channels][128 B], then the X ring
-  // x_full[kTcStagesMax] x_empty[kTcStagesMax] acc_full[2] acc_empty[2] done
-  uint64_t* bars = reinterpret_cast<uint64_t*>(base + kTcSlots * kTcXStageBytes);
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * kTcStagesMax + 5);
+  uint8_t* xsm = smem_raw + (((raw + 1023u) & ~1023u) - raw);  // [stage][atom][128 tokens][128 B], 1024-aligned
+  // x_full[kTcStages] x_empty[kTcStages] acc_full[2] acc_empty[2] done w_ready
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xsm + kTcStages * kTcXStageBytes);
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * kTcStages + 6);
   int* counters = reinterpret_cast<int*>(tmem_holder + 1);  // [0] tiles issued by TMA, [1] consumed by MMA, [2] fail
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -302,17 +312,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   const int ntiles = a.n_seqs * nrows;
   if (r == 0 || chunk >= ntiles) return;
   const int my_tiles = (ntiles - chunk + a.chunks - 1) / a.chunks;
-  const int nsplit = b >= 6 ? 3 : 2, nstage = kTcSlots - nsplit;
-  uint8_t* xsm = wsm + nsplit * kTcSplitBytes;  // [stage][atom][128 tokens][128 B]
+  const int nsplit = b >= 6 ? 3 : 2;
   const float* pool = param_pool(a.block);
-  const float* W = pool + he.w_off;
   const uint32_t bar0 = smem_addr(bars);
   auto bar = [&](int i) { return bar0 + 8u * i; };
-  const int XF = 0, XE = kTcStagesMax, AF = 2 * kTcStagesMax, AE = AF + 2, DONE = AF + 4;
+  const int XF = 0, XE = kTcStages, AF = 2 * kTcStages, AE = AF + 2, DONE = AF + 4, WREADY = AF + 5;
 
-  // ---- setup: barriers, TMEM, split basis ----
+  // ---- setup: barriers, TMEM ----
   if (tid == 0) {
-    for (int i = 0; i < nstage; ++i) {
+    for (int i = 0; i < kTcStages; ++i) {
       mbar_init(bar(XF + i), 1);  // producer arrive + TMA bytes
       mbar_init(bar(XE + i), 1);  // MMA commit
     }
@@ -320,56 +328,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       mbar_init(bar(AF + i), 1);  // MMA commit
       mbar_init(bar(AE + i), 4);  // one arrive per epilogue warp
     }
-    mbar_init(bar(DONE), 1);      // final MMA commit
+    mbar_init(bar(DONE), 1);    // final MMA commit
+    mbar_init(bar(WREADY), 4);  // one arrive per epilogue warp once its basis rows are in TMEM
     counters[0] = counters[1] = counters[2] = 0;
     fence_mbar_init();
   }
   if (warp == 1) tmem_alloc(smem_addr(tmem_holder), kTcTmemCols);
-  // W split terms of channel n, dims [64 atom + 8 c, +8): one 16-byte chunk per term, stored at
-  // chunk position c ^ (n & 7) of the term's swizzled row; channels n >= r are zero.  Each
-  // chunk of W is loaded once (two 16-byte loads), four chunks per thread in flight together.
-  {
-    constexpr int kChunks = 2 * 128 * 8;  // (atom, channel, c)
-#pragma unroll 1
-    for (int base = 0; base < kChunks; base += 4 * kTcThreads) {
-      float4 wv[4][2];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int idx = base + u * kTcThreads + tid;
-        const int c = idx & 7, n = (idx >> 3) & 127, atom = idx >> 10;
-        if (idx < kChunks && n < r) {
-          const float4* src = reinterpret_cast<const float4*>(W + (size_t)n * kD + 64 * atom + 8 * c);
-          wv[u][0] = src[0];
-          wv[u][1] = src[1];
-        } else {
-          wv[u][0] = wv[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int idx = base + u * kTcThreads + tid;
-        if (idx >= kChunks) break;
-        const int c = idx & 7, n = (idx >> 3) & 127, atom = idx >> 10;
-        float rem[8] = {wv[u][0].x, wv[u][0].y, wv[u][0].z, wv[u][0].w, wv[u][1].x, wv[u][1].y, wv[u][1].z, wv[u][1].w};
-        for (int sp = 0; sp < nsplit; ++sp) {
-          uint32_t packed[4];
-#pragma unroll
-          for (int e2 = 0; e2 < 4; ++e2) {
-            const float p0 = __bfloat162float(__float2bfloat16_rn(rem[2 * e2]));
-            const float p1 = __bfloat162float(__float2bfloat16_rn(rem[2 * e2 + 1]));
-            rem[2 * e2] -= p0;
-            rem[2 * e2 + 1] -= p1;
-            packed[e2] = pack_bf16(p0, p1);
-          }
-          uint8_t* rowp = wsm + (size_t)sp * kTcSplitBytes + (size_t)atom * 128 * 128 + (size_t)n * 128;
-          *reinterpret_cast<uint4*>(rowp + ((c ^ (n & 7)) << 4)) =
-              make_uint4(packed[0], packed[1], packed[2], packed[3]);
-        }
-      }
-    }
-  }
-  // generic-proxy writes of the basis must be visible to the tensor cores (async proxy)
-  fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -380,7 +344,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       int issued = 0;
       for (int i = 0; i < my_tiles; ++i) {
-        const int st = i % nstage, ph = (i / nstage) & 1;
+        const int st = i % kTcStages, ph = (i / kTcStages) & 1;
         if (!mbar_wait_bounded(bar(XE + st), ph ^ 1, kTcWaitNs)) {
           atomicOr(&g_status, 1u);
           counters[2] = 1;
@@ -389,11 +353,12 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         if (counters[2]) break;
         const int tile = chunk + i * a.chunks;
         const int seq = tile / nrows, row = tile % nrows;
-        int c[5] = {0, 0, 0, 0, 0};
-        c[a.slot_head] = kv;
-        c[a.slot_tok] = row * kRowTokens;
-        c[a.slot_seq] = seq;
-        c[a.slot_layer] = layer;
+        int c[5];
+        c[0] = 0;
+#pragma unroll
+        for (int d = 1; d < 5; ++d)
+          c[d] = (a.slot_head == d ? kv : 0) + (a.slot_tok == d ? row * kRowTokens : 0) + (a.slot_seq == d ? seq : 0) +
+                 (a.slot_layer == d ? layer : 0);
         mbar_arrive_expect_tx(bar(XF + st), kTcXStageBytes);
         const uint32_t dst = smem_addr(xsm + st * kTcXStageBytes);
         tma_load_5d(dst, &xmap, c, bar(XF + st));
@@ -407,11 +372,17 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // ---------------- MMA issuer: Y^T[128 channels][128 tokens] per tile ----------------
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_bf16(128, 128);
-      const uint32_t wbase = smem_addr(wsm), xbase = smem_addr(xsm);
+      const uint32_t xbase = smem_addr(xsm);
       int consumed = 0;
-      for (int i = 0; i < my_tiles; ++i) {
-        const int st = i % nstage, acc = i & 1;
-        if (!mbar_wait_bounded(bar(XF + st), (i / nstage) & 1, kTcWaitNs) ||
+      const bool w_ok = mbar_wait_bounded(bar(WREADY), 0, kTcWaitNs);
+      if (!w_ok) {
+        atomicOr(&g_status, 1u);
+        counters[2] = 1;
+      }
+      tc_fence_after();
+      for (int i = 0; w_ok && i < my_tiles; ++i) {
+        const int st = i % kTcStages, acc = i & 1;
+        if (!mbar_wait_bounded(bar(XF + st), (i / kTcStages) & 1, kTcWaitNs) ||
             !mbar_wait_bounded(bar(AE + acc), ((i >> 1) & 1) ^ 1, kTcWaitNs)) {
           atomicOr(&g_status, 1u);
           counters[2] = 1;
@@ -425,8 +396,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
             const uint32_t koff = (uint32_t)((kk >> 2) * 16384 + (kk & 3) * 32);
-            tc_mma_bf16(d, umma_desc_sw128(wbase + sp * kTcSplitBytes + koff),
-                        umma_desc_sw128(xbase + st * kTcXStageBytes + koff), idesc, (sp > 0 || kk > 0) ? 1u : 0u);
+            tc_mma_bf16_ts(d, tmem + (uint32_t)(kTcWCol + 64 * sp + 8 * kk),
+                           umma_desc_sw128(xbase + st * kTcXStageBytes + koff), idesc, (sp > 0 || kk > 0) ? 1u : 0u);
           }
         tc_commit(bar(XE + st));   // X stage free once these MMAs completed
         tc_commit(bar(AF + acc));  // accumulator ready
@@ -438,12 +409,47 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else {
     // ---------------- epilogue (warps 2..5): one channel per thread ----------------
     const int ch = 32 * (warp & 3) + lane;
+    const uint32_t tq = tmem + ((uint32_t)(32 * (warp & 3)) << 16);  // this warp's TMEM lane quarter
+    // Basis row of channel ch as nsplit bf16 terms, the A operand of the MMAs: TMEM lane ch,
+    // column kTcWCol + 64 sp + c holds dims 2c (low half) and 2c + 1 of term sp; rows of
+    // channels >= r are zero.
+    {
+      const float4* wrow = reinterpret_cast<const float4*>(pool + he.w_off + (size_t)(ch < r ? ch : 0) * kD);
+#pragma unroll 1
+      for (int q = 0; q < 4; ++q) {
+        float rem[32];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const float4 f = ch < r ? wrow[8 * q + u] : make_float4(0.f, 0.f, 0.f, 0.f);
+          rem[4 * u] = f.x;
+          rem[4 * u + 1] = f.y;
+          rem[4 * u + 2] = f.z;
+          rem[4 * u + 3] = f.w;
+        }
+#pragma unroll 1
+        for (int sp = 0; sp < nsplit; ++sp) {
+          uint32_t packed[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const float p0 = __bfloat162float(__float2bfloat16_rn(rem[2 * c]));
+            const float p1 = __bfloat162float(__float2bfloat16_rn(rem[2 * c + 1]));
+            rem[2 * c] -= p0;
+            rem[2 * c + 1] -= p1;
+            packed[c] = pack_bf16(p0, p1);
+          }
+          tc_st32x16(tq + (uint32_t)(kTcWCol + 64 * sp + 16 * q), packed);
+        }
+      }
+      tc_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(bar(WREADY));
+    }
     TcEpi e;
     const float scale = 1.0f / (float)(1 << b);  // a power of two: the scaled values are exact
     e.inv_s = he.inv_delta * scale;
     e.cterm_s = ((float)(1 << (b - 1)) - (ch < r ? pool[he.wmu_off + ch] : 0.f) * he.inv_delta) * scale;
     e.top = kTcMagicBits + (1u << b) - 1u;
-    const uint32_t tq = tmem + ((uint32_t)(32 * (warp & 3)) << 16);  // this warp's TMEM lane quarter
     switch (b) {
       case 1: tc_epilogue<1>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
       case 2: tc_epilogue<2>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
@@ -459,7 +465,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   __syncthreads();
   if (tid == 0) {
     for (int i = counters[1]; i < counters[0]; ++i)
-      if (!mbar_wait_bounded(bar(XF + i % nstage), (i / nstage) & 1, kTcWaitNs)) break;
+      if (!mbar_wait_bounded(bar(XF + i % kTcStages), (i / kTcStages) & 1, kTcWaitNs)) break;
   }
   tc_fence_before();
   __syncthreads();
