@@ -34,6 +34,7 @@ sys.path.insert(0, ROOT)
 METRIC = "decode-attn effective HBM GB/s over packed cache (% of peak); compress tok/s"
 FALLBACK_HBM_GBS = 6800.0
 PROFILE = os.path.join(ROOT, "profiles", "decode_scan_llama3_8b.txt")
+CONFIG3_PROFILE = os.path.join(ROOT, "profiles", "decode_scan_llama3_70b_joint.txt")
 SCAN_SOURCES = ["paper_2609_24298_gb300/csrc/decode.cuh", "paper_2609_24298_gb300/csrc/common.cuh"]
 CFG = 2
 SAMPLE_R, SAMPLE_B = 64, 2  # (r, b) of the oracle sample heads: the most common point at 1 bpd
@@ -806,6 +807,7 @@ def run_config3_leg(args, dev, stream, cpu_baseline: bool):
     out, _ = workload_leg(args, dev, stream, 3, spec["bpd"], [spec["tokens"]], False, args.config_steps,
                           cpu_baseline, label="llama3-70b-shaped decode step: 80 layers x 8 kv heads (GQA 8) x 1 "
                                               "sequence x 131072 tokens, K and V allocated jointly at 0.5 bpd")
+    out["roofline"]["traffic"] = profiled_traffic(CONFIG3_PROFILE, SCAN_SOURCES)
     return out
 
 
