@@ -101,6 +101,39 @@ def test_compress_seqs_offset_and_paged():
             check_head(host, offs[h], 1, p, xs[q, :, h], T, t0=t0, seq=q, page_table=pt)
 
 
+def test_compress_clamps_at_both_ends():
+    """Tokens scaled by 0, +-40 and +-400 push y / Delta far outside [-2^{b-1}, 2^{b-1}) for
+    every bit width: wherever the oracle's pre-rounding value u lies outside [-0.5, 2^b + 0.5]
+    the code must be exactly 0 or 2^b - 1, the zero tokens must give the code of the mean's
+    projection, and the rest may differ by one near a cell boundary (the scaled inputs scale
+    the rounding error of the projection with them).  The packed bytes must re-pack exactly."""
+    srcs = [synth.HeadSource(17, 0, i, 0, (0.5, 2.0)) for i in range(8)]
+    params = [oracle_head(s, 16 * (1 + i % 3), i + 1) for i, s in enumerate(srcs)]
+    T = 260
+    scale = np.array([0.0, 1.0, 40.0, -40.0, 400.0, -400.0, 0.5, -1.0])[np.arange(T) % 8]
+    xs = np.stack([s.tokens(T) for s in srcs], axis=1)[None] * scale[None, :, None, None]
+    xs = torch.tensor(xs).to(torch.bfloat16).double().numpy()  # the values the kernel reads
+    host, offs, r, b, xs = run_compress(params, srcs, T, 0, x_override=xs)
+    saturated = 0
+    for h, p in enumerate(params):
+        r_, b_ = p["r"], p["b"]
+        got = read_head_codes(host, offs[h], 0, r_, b_, T)
+        u, want = ocomp.compress(xs[0, :, h], p["W"], p["mu"], p["delta"], b_)
+        outside = (u < -0.5) | (u > (1 << b_) + 0.5)
+        assert np.array_equal(got[outside], want[outside]), (r_, b_)
+        assert np.all(np.abs(got - want) <= 1), (r_, b_)
+        zero = scale == 0.0
+        assert codes_ok(got[zero], u[zero], want[zero]), (r_, b_)
+        saturated += int(outside.sum())
+        for row in range(-(-T // 128)):
+            addr = olay.row_address(int(offs[h]), r_, b_, 0, row, -(-T // 128), None)
+            codes = np.zeros((128, r_), np.int64)
+            lo, hi = row * 128, min((row + 1) * 128, T)
+            codes[: hi - lo] = got[lo:hi]
+            assert np.array_equal(olay.pack_row(codes, 0, b_), host[addr:addr + olay.row_bytes(r_, b_)]), (r_, b_, row)
+    assert saturated > 2000  # both clamps were exercised
+
+
 def test_compress_zero_rank_head_writes_nothing():
     srcs = [synth.HeadSource(14, 0, i, 0, (0.5, 2.0)) for i in range(2)]
     params = [oracle_head(srcs[0], 0, 1), oracle_head(srcs[1], 16, 4)]
