@@ -573,7 +573,8 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
   };
   for (int item = take(); item < n_items && !w.failed; item = take()) {
     if constexpr (G == 4) {
-      // the bit widths of 1 to 3 that carry most of the cache at low rates get their own code
+      // the bit widths of 1 to 3 that carry most of the cache at low rates, and the 3- to 5-bit
+      // pairs of rates of 3 to 4 bpd, get their own code
       const WsGroup gr = groups[items[item].group];
       const HeadEntry hk = heads[gr.k_head], hv = heads[gr.v_head];
       const int key = (hk.r > 0 ? hk.b : 0) * 16 + (hv.r > 0 ? hv.b : 0);
@@ -587,6 +588,12 @@ __global__ void __launch_bounds__(kDecodeWarps * 32, 4) decode_kernel(DecodeArgs
         case 0x31: scan_item<G, 3, 1>(a, w, item); break;
         case 0x32: scan_item<G, 3, 2>(a, w, item); break;
         case 0x33: scan_item<G, 3, 3>(a, w, item); break;
+        case 0x34: scan_item<G, 3, 4>(a, w, item); break;
+        case 0x43: scan_item<G, 4, 3>(a, w, item); break;
+        case 0x44: scan_item<G, 4, 4>(a, w, item); break;
+        case 0x45: scan_item<G, 4, 5>(a, w, item); break;
+        case 0x54: scan_item<G, 5, 4>(a, w, item); break;
+        case 0x55: scan_item<G, 5, 5>(a, w, item); break;
         default: scan_item<G, 0, 0>(a, w, item); break;
       }
     } else {

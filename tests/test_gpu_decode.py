@@ -113,7 +113,9 @@ def test_tiny_config_full():
     assert rel_err(o, ref) < TOL
 
 
-@pytest.mark.parametrize("bk,bv", [(1, 8), (2, 7), (3, 6), (4, 5), (5, 4), (6, 3), (7, 2), (8, 1)])
+# every width on each side, plus the pairs whose item loops have their own code at G = 4
+@pytest.mark.parametrize("bk,bv", [(1, 8), (2, 7), (3, 6), (4, 5), (5, 4), (6, 3), (7, 2), (8, 1),
+                                   (3, 4), (4, 3), (4, 4), (5, 5)])
 def test_every_bit_width(bk, bv):
     rbs = [(128 if bk <= 2 else 48, bk), (18, bk), (128 if bv <= 2 else 40, bv), (2, bv)]
     params, srcs = mixed_heads(2, rbs, cfg=32 + bk)
