@@ -4,7 +4,7 @@
 //
 // One CTA per (layer, kv head) and chunk of 128-token tiles, 6 warps:
 //   warp 0    TMA producer: each tile X [128 tokens x 128 dims] bf16 arrives as two 64-dim
-//             boxes with 128-byte swizzle into a 7-stage shared-memory ring.
+//             boxes with 128-byte swizzle into a 6-stage shared-memory ring.
 //   warp 1    allocates TMEM; one thread issues tcgen05.mma computing the transposed
 //             projection Y^T = W X^T (M = 128 channels, rows past r zero; N = 128 tokens;
 //             K = 16 per instruction; bf16 inputs, fp32 accumulation in TMEM).  The head's
@@ -38,8 +38,11 @@ constexpr int kTcEpiWarp0 = 2;
 constexpr int kTcTmemCols = 512;
 constexpr int kTcWCol = 256;
 constexpr int kTcXStageBytes = 2 * 16384;  // two 64-dim swizzle atoms of 128 rows
-constexpr int kTcStages = 7;               // X ring
-constexpr int kTcSmemBytes = 1024 + kTcStages * kTcXStageBytes + 256;
+constexpr int kTcStages = 6;               // X ring
+constexpr int kTcRowStage = 16 * 128 * 8;  // one code row of the widest head (r = 128, b = 8)
+// X ring, then two code-row staging buffers (the bulk store of one tile's row reads its buffer
+// while the next tile's row is written into the other)
+constexpr int kTcSmemBytes = 1024 + kTcStages * kTcXStageBytes + 2 * kTcRowStage + 256;
 
 struct TcArgs {
   const unsigned char* block;
@@ -121,6 +124,35 @@ __device__ __forceinline__ void tc_wait_ld(uint32_t (&v)[32]) {
 }
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+// shared -> global bulk store of `bytes` (a multiple of 16, both addresses 16-byte aligned),
+// committed as its own bulk group
+__device__ __forceinline__ void bulk_store_s2g(void* dst, uint32_t src, uint32_t bytes) {
+  asm volatile(
+      "cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n"
+      "cp.async.bulk.commit_group;" ::"l"(dst),
+      "r"(src), "r"(bytes)
+      : "memory");
+}
+// wait until at most one bulk group of this thread is still reading its shared-memory source
+__device__ __forceinline__ void bulk_store_wait_read_1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+// wait until every bulk group of this thread has completed
+__device__ __forceinline__ void bulk_store_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// named barrier `id` over the four epilogue warps
+__device__ __forceinline__ void tc_epi_sync(int id) {
+  asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory");
+}
+// the same barrier, returning whether `p` holds in all four warps
+__device__ __forceinline__ bool tc_epi_all(int id, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.b32 p, %1, 0;\n bar.red.and.pred q, %2, 128, p;\n selp.u32 %0, 1, 0, q;\n}\n"
+      : "=r"(r)
+      : "r"((int)p), "r"(id)
+      : "memory");
+  return r != 0;
 }
 
 // Shared-memory matrix descriptor of a K-major operand in the 128-byte swizzled canonical
@@ -223,16 +255,21 @@ __device__ __forceinline__ void tc_row_words(const uint32_t (&sub)[8][(B + 1) / 
 template <int B>
 __device__ __forceinline__ void tc_epilogue(const TcArgs& a, const HeadEntry& he, const TcEpi& e, int chunk,
                                             int my_tiles, int nrows, uint32_t tmem_q, uint32_t bar_acc_full,
-                                            uint32_t bar_acc_empty, int* fail) {
+                                            uint32_t bar_acc_empty, uint8_t* rsm, int* fail) {
   constexpr int NW = (B + 1) / 2;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int ch = 32 * (warp & 3) + lane;  // this thread's channel = its TMEM lane
   const uint32_t rb = 16u * he.r * B;
+  // the first epilogue thread issues the bulk stores of the code rows
+  const bool issuer = threadIdx.x == 32 * kTcEpiWarp0;
   for (int i = 0; i < my_tiles; ++i) {
     const int acc = i & 1;
     const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(bar_acc_full + 8u * acc, (i >> 1) & 1, kTcWaitNs));
-    if (!ok) {
-      if (lane == 0) {
+    // the row staging buffer of tile i is free once the bulk store of tile i - 2 has read it
+    if (issuer) bulk_store_wait_read_1();
+    // every epilogue warp meets here once per tile; a failed wait in any of them stops all four
+    if (!tc_epi_all(1, ok)) {
+      if (lane == 0 && !ok) {
         atomicOr(&g_status, 1u);
         *fail = 1;
       }
@@ -283,14 +320,24 @@ __device__ __forceinline__ void tc_epilogue(const TcArgs& a, const HeadEntry& he
     }
     uint32_t words[4 * B];
     tc_row_words<B>(sub, a.side, lane, words);
+    uint8_t* stg = rsm + (size_t)(i & 1) * kTcRowStage;
     if (ch < he.r) {
-      uint8_t* dst = a.cache + row_offset(he.cache_off, rb, seq, (a.t0 >> 7) + row, a.page_table, a.pages_per_seq,
-                                          a.rows_per_seq) + (size_t)ch * 16 * B;
 #pragma unroll
       for (int k = 0; k < B; ++k)
-        reinterpret_cast<uint4*>(dst)[k] = make_uint4(words[4 * k], words[4 * k + 1], words[4 * k + 2], words[4 * k + 3]);
+        reinterpret_cast<uint4*>(stg + (size_t)ch * 16 * B)[k] =
+            make_uint4(words[4 * k], words[4 * k + 1], words[4 * k + 2], words[4 * k + 3]);
+    }
+    // the generic-proxy writes of the row must be visible to the bulk copy (async proxy)
+    fence_proxy_async_smem();
+    tc_epi_sync(2);
+    if (issuer) {
+      uint8_t* dst = a.cache + row_offset(he.cache_off, rb, seq, (a.t0 >> 7) + row, a.page_table, a.pages_per_seq,
+                                          a.rows_per_seq);
+      bulk_store_s2g(dst, smem_addr(stg), rb);
     }
   }
+  // every row written and the staging buffers read before the CTA's shared memory goes away
+  if (issuer) bulk_store_wait_all();
 }
 
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -298,8 +345,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* xsm = smem_raw + (((raw + 1023u) & ~1023u) - raw);  // [stage][atom][128 tokens][128 B], 1024-aligned
+  uint8_t* rsm = xsm + kTcStages * kTcXStageBytes;  // [2][kTcRowStage] code rows on their way out
   // x_full[kTcStages] x_empty[kTcStages] acc_full[2] acc_empty[2] done w_ready
-  uint64_t* bars = reinterpret_cast<uint64_t*>(xsm + kTcStages * kTcXStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(rsm + 2 * kTcRowStage);
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(bars + 2 * kTcStages + 6);
   int* counters = reinterpret_cast<int*>(tmem_holder + 1);  // [0] tiles issued by TMA, [1] consumed by MMA, [2] fail
 
@@ -451,14 +499,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     e.cterm_s = ((float)(1 << (b - 1)) - (ch < r ? pool[he.wmu_off + ch] : 0.f) * he.inv_delta) * scale;
     e.top = kTcMagicBits + (1u << b) - 1u;
     switch (b) {
-      case 1: tc_epilogue<1>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      case 2: tc_epilogue<2>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      case 3: tc_epilogue<3>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      case 4: tc_epilogue<4>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      case 5: tc_epilogue<5>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      case 6: tc_epilogue<6>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      case 7: tc_epilogue<7>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
-      default: tc_epilogue<8>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), &counters[2]); break;
+      case 1: tc_epilogue<1>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      case 2: tc_epilogue<2>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      case 3: tc_epilogue<3>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      case 4: tc_epilogue<4>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      case 5: tc_epilogue<5>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      case 6: tc_epilogue<6>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      case 7: tc_epilogue<7>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
+      default: tc_epilogue<8>(a, he, e, chunk, my_tiles, nrows, tq, bar(AF), bar(AE), rsm, &counters[2]); break;
     }
   }
   // ---- teardown: drain the TMA loads nobody consumed, then free TMEM ----
