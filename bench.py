@@ -127,7 +127,8 @@ class ClockSampler:
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,"
+              "clocks.mem,temperature.gpu")
 
     def __init__(self, index: int):
         self.index = index
@@ -152,7 +153,7 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except subprocess.TimeoutExpired:
             self.proc.kill()
-        sm, smax, reasons = [], [], set()
+        sm, smax, mem, temp, reasons = [], [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in open(self.path):
             parts = [p.strip() for p in line.split(",")]
@@ -166,9 +167,19 @@ class ClockSampler:
             for n, v in zip(names, parts[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(n)
+            try:
+                mem.append(float(parts[9]))
+                temp.append(float(parts[10]))
+            except (IndexError, ValueError):
+                pass
         os.unlink(self.path)
-        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(smax) if smax else None,
-                "samples": len(sm), "reasons": sorted(reasons)}
+        out = {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+               "samples": len(sm), "reasons": sorted(reasons)}
+        if mem:
+            out["mem_mhz"] = float(np.median(mem))
+        if temp:
+            out["gpu_temp_c"] = float(np.median(temp))
+        return out
 
 
 # ---------------------------------------------------------------------------------------
@@ -340,12 +351,15 @@ def run_compress_leg(args, dev, stream, peak):
         raise RuntimeError("device status after compress warm-up")
     K = max(5, min(50, args.steps // 40))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(dev.index if dev.index is not None else 0)
     torch.cuda.synchronize()
+    clocks.start()
     e0.record(stream)
     for _ in range(K):
         one_pass()
     e1.record(stream)
     torch.cuda.synchronize()
+    clk = clocks.stop()
     if cobra.cobra_check(stream) != cobra.COBRA_OK:
         raise RuntimeError("device status after the compress timed region")
     ms = e0.elapsed_time(e1) / K
@@ -367,6 +381,7 @@ def run_compress_leg(args, dev, stream, peak):
                      "traffic_per_launch": traffic if L == 32 else None,
                      "tensor_tflops_algorithmic": flops / (ms * 1e-3) / 1e12},
         "l2": f"inputs larger than L2 ({in_bytes / 1e9:.1f} GB of bf16 K/V read every pass)",
+        "clocks": clk,
     }
 
 
