@@ -340,8 +340,9 @@ cobra_status cobra_decode_qproj_append(const void* params, const cobra_decode_de
  * at pos[s] (Table alg:kvrobin step 7), then decode attention over seq_lens[s] tokens (which
  * normally include the appended one).  kdesc / vdesc describe the K / V heads of `desc`
  * (sides 0 / 1, head0 = desc->k_head0 / desc->v_head0, the other counts equal, else
- * COBRA_EINVAL).  Four launches on `stream`: V append, query projection with the K append,
- * scan, combine; nothing is synchronised.  k_new, v_new, q and out may live in pinned host
+ * COBRA_EINVAL).  Three launches on `stream`: the query projection with both appends (its
+ * grid carries one CTA per (layer, kv head) for the projection and K append, and one for the
+ * V append), the scan, the combine; nothing is synchronised.  k_new, v_new, q and out may live in pinned host
  * memory (any memory the device can address): the kernels then read and write it in place. */
 cobra_status cobra_decode_step(const void* params, const cobra_decode_desc* desc, const cobra_decode_info* info,
                                const cobra_compress_desc* kdesc, const cobra_compress_desc* vdesc, const void* k_new,

@@ -156,14 +156,15 @@ __device__ __forceinline__ void append_tokens(const CompressArgs& a, const HeadE
   }
 }
 
-__global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) {
-  extern __shared__ __align__(16) float apsm[];
+// The append of (layer, kv head) number `blk` by one CTA of kAppendThreads threads, with
+// append_smem_bytes() of shared memory at apsm.  Run by append_kernel and, in the decode step,
+// by the V-side CTAs of the query projection's launch.
+__device__ __forceinline__ void append_block(const CompressArgs& a, int blk, float* apsm) {
   float* Ws = apsm;                     // [kD][kAppendWLd]
   const int warp = threadIdx.x >> 5;
   float* wmu = Ws + kD * kAppendWLd + (kAppendThreads / 32) * kD;  // W^T mu
   float* xs = Ws + kD * kAppendWLd + warp * kD;
-  grid_dep_launch();
-  const int layer = blockIdx.x / a.n_kv, kv = blockIdx.x % a.n_kv;
+  const int layer = blk / a.n_kv, kv = blk % a.n_kv;
   const HeadEntry he = head_table(a.block)[a.head0 + layer * a.layer_stride + kv];
   if (he.r == 0) {
     grid_dep_wait();
@@ -181,6 +182,12 @@ __global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) 
   cp_async_wait_all();
   __syncthreads();
   append_tokens(a, he, layer, kv, Ws, wmu, xs, warp, kAppendThreads / 32, nx);
+}
+
+__global__ void __launch_bounds__(kAppendThreads) append_kernel(CompressArgs a) {
+  extern __shared__ __align__(16) float apsm[];
+  grid_dep_launch();
+  append_block(a, blockIdx.x, apsm);
 }
 
 }  // namespace cobra

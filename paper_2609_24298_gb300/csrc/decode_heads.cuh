@@ -26,6 +26,7 @@ __host__ __device__ constexpr int combine_zld() {
 __host__ __device__ constexpr size_t qproj_smem_bytes() {
   return sizeof(float) * ((size_t)kD * kWLd + (size_t)kVecPass * kD + (size_t)kVecPass * kWLd + kD);
 }
+static_assert(append_smem_bytes() <= qproj_smem_bytes(), "the V-append CTAs use the projection's shared memory");
 static_assert(kWLd == kAppendWLd, "the query projection stages W_K as the append reads it");
 constexpr int kWtChunk = 64;  // chunk weights held in shared memory per vector and round
 constexpr int kCombineVP = 16;  // query vectors per combine CTA (a head's sequences spread over CTAs)
@@ -40,11 +41,20 @@ __host__ __device__ constexpr size_t combine_smem_bytes() {
 //   that max |q~| of the group lands in [256, 512), split into fp16 hi + lo and laid out as
 //   the scan's MMA B fragments; Qsum_g = sum over channels of the fed hi + lo values.
 //   With ak.x set, the CTA first appends the new K token of every sequence of its head (a8),
-//   which projects through the same staged W_K.
+//   which projects through the same staged W_K.  With av.x set, the grid has a second half of
+//   CTAs (blockIdx.x >= n_qblocks) that append the new V tokens, one (layer, kv head) each, so
+//   that both appends and the projection run in one launch.
 // ---------------------------------------------------------------------------------------
+static_assert(kAppendThreads == kHeadThreads, "the V append runs in the query projection's CTAs");
 template <int G>
-__global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a, CompressArgs ak) {
+__global__ void __launch_bounds__(kHeadThreads) qproj_kernel(DecodeArgs a, CompressArgs ak, CompressArgs av,
+                                                             int n_qblocks) {
   grid_dep_launch();
+  if ((int)blockIdx.x >= n_qblocks) {
+    extern __shared__ __align__(16) float vsm[];
+    append_block(av, (int)blockIdx.x - n_qblocks, vsm);
+    return;
+  }
   constexpr int NTK = Heads<G>::NTK, SPP = kVecPass / G;
   extern __shared__ __align__(16) float qsm[];
   float* Ws = qsm;                  // [kD][kWLd]   W_K row i = channel i

@@ -257,7 +257,8 @@ enum Stage { kQproj = 1, kScan = 2, kCombine = 4 };
 
 template <int G>
 cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_items, int stages, cudaStream_t s,
-                           bool after_plan_kernel = false, const CompressArgs& ak = CompressArgs{}) {
+                           bool after_plan_kernel = false, const CompressArgs& ak = CompressArgs{},
+                           const CompressArgs& av = CompressArgs{}) {
   static Granted qproj_granted, combine_granted;
   if (ensure_smem(qproj_kernel<G>, qproj_smem_bytes(), qproj_granted) != COBRA_OK ||
       ensure_smem(combine_kernel<G, kCombineVP>, combine_smem_bytes<kCombineVP>(), combine_granted) != COBRA_OK)
@@ -265,10 +266,12 @@ cobra_status launch_decode(const DecodeArgs& a, int n_heads, int n_seqs, int n_i
   if (stages & kQproj) {
     // the query projection reads the plan before its wait; right after the plan kernel it is
     // launched in plain stream order
+    // with a V append, its CTAs follow the projection's (one per (layer, kv head))
+    const unsigned grid = (unsigned)n_heads * (av.x ? 2u : 1u);
     if (after_plan_kernel) {
-      qproj_kernel<G><<<n_heads, kHeadThreads, qproj_smem_bytes(), s>>>(a, ak);
+      qproj_kernel<G><<<grid, kHeadThreads, qproj_smem_bytes(), s>>>(a, ak, av, n_heads);
       if (cudaGetLastError() != cudaSuccess) return COBRA_ECUDA;
-    } else if (launch_pdl(qproj_kernel<G>, (unsigned)n_heads, kHeadThreads, qproj_smem_bytes(), s, a, ak) !=
+    } else if (launch_pdl(qproj_kernel<G>, grid, kHeadThreads, qproj_smem_bytes(), s, a, ak, av, n_heads) !=
                cudaSuccess) {
       return COBRA_ECUDA;
     }
@@ -343,15 +346,15 @@ cobra_status decode_args(const void* params, const cobra_decode_desc* d, const c
 cobra_status decode_common(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info, const void* q,
                            const uint8_t* cache, const int* seq_lens, const int* page_table, float* out,
                            void* workspace, size_t ws_bytes, void* stream, int stages,
-                           const CompressArgs& ak = CompressArgs{}) {
+                           const CompressArgs& ak = CompressArgs{}, const CompressArgs& av = CompressArgs{}) {
   DecodeArgs a;
   const cobra_status st =
       decode_args(params, d, info, q, cache, seq_lens, page_table, out, workspace, ws_bytes, stages, a);
   if (st != COBRA_OK) return st;
   cudaStream_t s = (cudaStream_t)stream;
   const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
-  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak);
-  return launch_decode<8>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak);
+  if (d->group == 4) return launch_decode<4>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak, av);
+  return launch_decode<8>(a, (int)n_heads, d->n_seqs, info->n_items, stages, s, false, ak, av);
 }
 
 // K-side append arguments that match the decode descriptor's K heads
@@ -407,10 +410,9 @@ extern "C" cobra_status cobra_decode_step(const void* params, const cobra_decode
   if (vdesc->side != 1 || vdesc->head0 != d->v_head0 || vdesc->layer_stride != d->layer_stride ||
       vdesc->n_layers != d->n_layers || vdesc->n_kv_heads != d->n_kv_heads || vdesc->n_seqs != d->n_seqs)
     return COBRA_EINVAL;
-  st = cobra_append(params, vdesc, v_new, pos, cache, page_table, stream);
-  if (st != COBRA_OK) return st;
+  // the V append runs in the query projection's launch (its second half of CTAs)
   return decode_common(params, d, info, q, cache, seq_lens, page_table, out, workspace, ws_bytes, stream,
-                       kQproj | kScan | kCombine, ak);
+                       kQproj | kScan | kCombine, ak, av);
 }
 
 extern "C" cobra_status cobra_decode_scan(const void* params, const cobra_decode_desc* d, const cobra_decode_info* info,
