@@ -344,16 +344,21 @@ def run_compress_leg(args, dev, stream, peak):
         for side in (0, 1):
             cobra.cobra_compress(dp.block, descs[side], xs[side], 0, T, dp.cache, None, stream)
 
-    for _ in range(3):
+    # the clock sampler's first readings take a moment: it starts with the warm-up, which keeps
+    # the GPU busy for about a second, so its samples are all taken under load
+    clocks = ClockSampler(dev.index if dev.index is not None else 0)
+    clocks.start()
+    t_start = time.time()
+    n_warm = 0
+    while n_warm < 3 or time.time() - t_start < 1.0:
         one_pass()
-    torch.cuda.synchronize()
+        torch.cuda.synchronize()
+        n_warm += 1
     if cobra.cobra_check(stream) != cobra.COBRA_OK:
+        clocks.stop()
         raise RuntimeError("device status after compress warm-up")
     K = max(5, min(50, args.steps // 40))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    clocks = ClockSampler(dev.index if dev.index is not None else 0)
-    torch.cuda.synchronize()
-    clocks.start()
     e0.record(stream)
     for _ in range(K):
         one_pass()
