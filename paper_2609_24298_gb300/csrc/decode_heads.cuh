@@ -299,19 +299,22 @@ __global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) 
     __syncthreads();
     // (2) zbar[v][i] = Delta (sum_k w_k acc_k[i] - 2^{b-1} + 1/2) with w_k = 2^(m_k - m*) / l*.
     //     Rounds of kWtChunk chunks (the first round's weights come from (1); later rounds
-    //     compute them one (vector, chunk) per thread into shared memory).  Thread (channel i,
-    //     group grp) of rw = r_V rounded up to 32, 64 or 128 channels owns the vectors
-    //     grp, grp + ng, ... (ng = 256 / rw groups) and sums over the chunks in blocks of
-    //     4 vectors x 8 chunks whose 32 loads are all issued before any is used.
+    //     compute them one (vector, chunk) per thread into shared memory).  Thread (channel
+    //     quad cq, slot) of rw = r_V rounded up to 32, 64 or 128 channels holds channels
+    //     4 cq .. 4 cq + 3 of the vectors slot, slot + ns, ... (ns = 256 / (rw / 4) slots) and
+    //     sums over the chunks in blocks of 8, the 16-byte loads of all its vectors' 8 chunks
+    //     issued before any is used.
     {
+      constexpr int VPT = (VP + 7) / 8;  // vectors per thread at most (ns >= 8)
       const int rw = rv <= 32 ? 32 : rv <= 64 ? 64 : kD;
-      const int ng = kHeadThreads / rw;
-      const int i = tid % rw, grp = tid / rw;
+      const int nq = rw / 4, ns = kHeadThreads / nq;
+      const int cq = tid % nq, slot = tid / nq;
+      const int pstride = wh->part_stride;
       int kmax = 0;
       for (int v = 0; v < nv; ++v) kmax = max(kmax, vinfo_n[v]);
-      float acc[VP / 2];
+      float4 acc[VPT];
 #pragma unroll
-      for (int q = 0; q < VP / 2; ++q) acc[q] = 0.f;
+      for (int q = 0; q < VPT; ++q) acc[q] = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int k0 = 0; k0 < kmax; k0 += kWtChunk) {
         if (k0 > 0) {
           __syncthreads();  // the previous round's weights are consumed
@@ -319,49 +322,57 @@ __global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) 
             const int v = idx / kWtChunk, k = k0 + idx % kWtChunk;
             float w = 0.f;
             if (k < vinfo_n[v]) {
-              const float mk = parts[(size_t)(vinfo_first[v] + k) * wh->part_stride + vinfo_g[v] * wh->g_stride];
+              const float mk = parts[(size_t)(vinfo_first[v] + k) * pstride + vinfo_g[v] * wh->g_stride];
               if (mk != -INFINITY) w = exp2f(mk - vinfo_m[v]) * vinfo_inv_l[v];
             }
             wts[idx] = w;
           }
           __syncthreads();
         }
-        if (i >= rv) continue;
+        if (4 * cq >= rv) continue;
         const int kr = min(kWtChunk, kmax - k0);
+        for (int kb = 0; kb < kr; kb += 8) {
+          float4 x[VPT][8];
 #pragma unroll
-        for (int q0 = 0; q0 < VP / 2; q0 += 4) {
-          if (grp + ng * q0 >= nv) break;
-          for (int kb = 0; kb < kr; kb += 8) {
-            float x[4][8];
+          for (int q = 0; q < VPT; ++q) {
+            const int v = slot + ns * q;
+            const int n = v < nv ? vinfo_n[v] - k0 : 0;
+            // the partial's channels start 4 floats in and every stride is a multiple of 4 floats
+            const float4* px = reinterpret_cast<const float4*>(
+                parts + (size_t)max(vinfo_first[v < nv ? v : 0], 0) * pstride + (size_t)k0 * pstride +
+                (v < nv ? vinfo_g[v] : 0) * wh->g_stride + 4 + 4 * cq);
 #pragma unroll
-            for (int qq = 0; qq < 4; ++qq) {
-              const int v = grp + ng * (q0 + qq);
-              const int n = v < nv ? vinfo_n[v] - k0 : 0;
-              const float* px = parts + (size_t)max(vinfo_first[v < nv ? v : 0], 0) * wh->part_stride +
-                                (size_t)k0 * wh->part_stride + (v < nv ? vinfo_g[v] : 0) * wh->g_stride + 4 + i;
+            for (int kk = 0; kk < 8; ++kk)
+              x[q][kk] = (kb + kk < n) ? px[(size_t)(kb + kk) * (pstride / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
 #pragma unroll
-              for (int kk = 0; kk < 8; ++kk) x[qq][kk] = (kb + kk < n) ? px[(size_t)(kb + kk) * wh->part_stride] : 0.f;
-            }
+          for (int q = 0; q < VPT; ++q) {
+            const int v = slot + ns * q;
+            if (v >= nv) break;
+            const float* wv = wts + v * kWtChunk + kb;
 #pragma unroll
-            for (int qq = 0; qq < 4; ++qq) {
-              const int v = grp + ng * (q0 + qq);
-              if (v >= nv) break;
-              const float* wv = wts + v * kWtChunk + kb;
-#pragma unroll
-              for (int kk = 0; kk < 8; ++kk) {
-                const float w = (kb + kk < kWtChunk) ? wv[kk] : 0.f;
-                acc[q0 + qq] += w != 0.f ? w * x[qq][kk] : 0.f;
+            for (int kk = 0; kk < 8; ++kk) {
+              const float w = (kb + kk < kWtChunk) ? wv[kk] : 0.f;
+              if (w != 0.f) {  // an empty chunk's value entries were never written
+                acc[q].x += w * x[q][kk].x;
+                acc[q].y += w * x[q][kk].y;
+                acc[q].z += w * x[q][kk].z;
+                acc[q].w += w * x[q][kk].w;
               }
             }
           }
         }
       }
-      if (i < rv) {
+      if (4 * cq < rv) {
 #pragma unroll
-        for (int q = 0; q < VP / 2; ++q) {
-          const int v = grp + ng * q;
+        for (int q = 0; q < VPT; ++q) {
+          const int v = slot + ns * q;
           if (v >= nv) break;
-          Zs[i * kZLd + v] = vinfo_first[v] >= 0 ? hv.delta * (acc[q] - cen) : 0.f;
+          const bool live = vinfo_first[v] >= 0;
+          const float a4[4] = {acc[q].x, acc[q].y, acc[q].z, acc[q].w};
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+            if (4 * cq + c < rv) Zs[(4 * cq + c) * kZLd + v] = live ? hv.delta * (a4[c] - cen) : 0.f;
         }
       }
     }
