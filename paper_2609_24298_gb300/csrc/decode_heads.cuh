@@ -302,10 +302,11 @@ __global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) 
     //     compute them one (vector, chunk) per thread into shared memory).  Thread (channel
     //     quad cq, slot) of rw = r_V rounded up to 32, 64 or 128 channels holds channels
     //     4 cq .. 4 cq + 3 of the vectors slot, slot + ns, ... (ns = 256 / (rw / 4) slots) and
-    //     sums over the chunks in blocks of 8, the 16-byte loads of all its vectors' 8 chunks
+    //     sums over the chunks in blocks of KB, the 16-byte loads of all its vectors' KB chunks
     //     issued before any is used.
     {
       constexpr int VPT = (VP + 7) / 8;  // vectors per thread at most (ns >= 8)
+      constexpr int KB = VPT >= 4 ? 4 : 8;  // chunks per block: VPT x KB 16-byte loads in flight
       const int rw = rv <= 32 ? 32 : rv <= 64 ? 64 : kD;
       const int nq = rw / 4, ns = kHeadThreads / nq;
       const int cq = tid % nq, slot = tid / nq;
@@ -331,8 +332,8 @@ __global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) 
         }
         if (4 * cq >= rv) continue;
         const int kr = min(kWtChunk, kmax - k0);
-        for (int kb = 0; kb < kr; kb += 8) {
-          float4 x[VPT][8];
+        for (int kb = 0; kb < kr; kb += KB) {
+          float4 x[VPT][KB];
 #pragma unroll
           for (int q = 0; q < VPT; ++q) {
             const int v = slot + ns * q;
@@ -342,7 +343,7 @@ __global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) 
                 parts + (size_t)max(vinfo_first[v < nv ? v : 0], 0) * pstride + (size_t)k0 * pstride +
                 (v < nv ? vinfo_g[v] : 0) * wh->g_stride + 4 + 4 * cq);
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
+            for (int kk = 0; kk < KB; ++kk)
               x[q][kk] = (kb + kk < n) ? px[(size_t)(kb + kk) * (pstride / 4)] : make_float4(0.f, 0.f, 0.f, 0.f);
           }
 #pragma unroll
@@ -351,7 +352,7 @@ __global__ void __launch_bounds__(kHeadThreads, 4) combine_kernel(DecodeArgs a) 
             if (v >= nv) break;
             const float* wv = wts + v * kWtChunk + kb;
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
+            for (int kk = 0; kk < KB; ++kk) {
               const float w = (kb + kk < kWtChunk) ? wv[kk] : 0.f;
               if (w != 0.f) {  // an empty chunk's value entries were never written
                 acc[q].x += w * x[q][kk].x;
