@@ -145,6 +145,13 @@ class ClockSampler:
         except OSError:
             self.proc = None
 
+    def has_sample(self) -> bool:
+        """Whether nvidia-smi has written its first reading (its first start can take seconds)."""
+        try:
+            return self.path is not None and os.path.getsize(self.path) > 0
+        except OSError:
+            return False
+
     def stop(self):
         if self.proc is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
@@ -344,13 +351,13 @@ def run_compress_leg(args, dev, stream, peak):
         for side in (0, 1):
             cobra.cobra_compress(dp.block, descs[side], xs[side], 0, T, dp.cache, None, stream)
 
-    # the clock sampler's first readings take a moment: it starts with the warm-up, which keeps
-    # the GPU busy for about a second, so its samples are all taken under load
+    # the clock sampler's first reading can take seconds: it starts with the warm-up, which keeps
+    # the GPU busy until that reading is in (at most 10 s), so its samples are all under load
     clocks = ClockSampler(dev.index if dev.index is not None else 0)
     clocks.start()
     t_start = time.time()
     n_warm = 0
-    while n_warm < 3 or time.time() - t_start < 1.0:
+    while n_warm < 3 or (time.time() - t_start < 10.0 and (time.time() - t_start < 1.0 or not clocks.has_sample())):
         one_pass()
         torch.cuda.synchronize()
         n_warm += 1
