@@ -353,7 +353,7 @@ def run_compress_leg(args, dev, stream, peak):
 
     # the clock sampler's first reading can take seconds: it starts with the warm-up, which keeps
     # the GPU busy until that reading is in (at most 10 s), so its samples are all under load
-    clocks = ClockSampler(dev.index if dev.index is not None else 0)
+    clocks = ClockSampler(torch.device(dev).index or 0)
     clocks.start()
     t_start = time.time()
     n_warm = 0
