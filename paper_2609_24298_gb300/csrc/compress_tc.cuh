@@ -20,6 +20,8 @@
 //             4 (channel parity) + (t/2) % 4, rho = t / 8, half = t % 2).  A lane then owns
 //             bytes [16 b i, 16 b (i + 1)) of the code row of its channel i: V rows from its
 //             own sub-streams, K rows after exchanging half of them with the partner channel.
+//             The lanes write their bytes into a shared-memory staging buffer, and after a
+//             barrier of the four warps one thread stores the whole row with a bulk copy.
 // All waits are bounded; on a timeout the kernel records it in the status word, drains the
 // copies and MMAs it issued, frees its TMEM and returns.
 #pragma once
