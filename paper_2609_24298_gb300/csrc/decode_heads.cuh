@@ -1,6 +1,7 @@
 // Per-head kernels of decode attention (Table alg:kvrobin step 8; App. G): the query
 // projection ahead of the scan of decode.cuh (optionally fused with the K-side append of one
-// new token, step 7) and the combine + back-projection after it.
+// new token, step 7, and carrying the V-side append's CTAs in the same launch) and the
+// combine + back-projection after it.
 #pragma once
 
 #include "compress.cuh"
@@ -9,9 +10,10 @@
 namespace cobra {
 
 // ---------------------------------------------------------------------------------------
-// Per-head kernels (query projection, combine): one CTA of 256 threads per (layer, kv head),
+// Per-head kernels: the query projection has one CTA of 256 threads per (layer, kv head),
 // looping over the sequences 32 query vectors at a time, with the head's basis staged in
-// shared memory once.  The workspace's head-group table gives the group of (head, seq).
+// shared memory once; the combine has one per (layer, kv head) and run of kCombineVP query
+// vectors.  The workspace's head-group table gives the group of (head, seq).
 // ---------------------------------------------------------------------------------------
 constexpr int kHeadThreads = 256;
 constexpr int kVecPass = 32;  // query vectors (sequences x G) per pass
