@@ -163,6 +163,17 @@ def test_peaked_queries_and_many_chunks():
     assert rel_err(o, ref) < TOL
 
 
+@pytest.mark.parametrize("G", [4, 8])
+def test_many_chunks_partial_channel_quads(G):
+    """The combine reads the chunk sums four channels at a time: V ranks that are not a
+    multiple of 4 (42, 6) leave a partly used last quad, over groups cut into many chunks."""
+    rbs = [(128, 2), (64, 3), (42, 2), (6, 3)]
+    params, srcs = mixed_heads(2, rbs, cfg=47)
+    o, ref, info = run_decode(params, srcs, 1, 2, G, [24000, 9000])
+    assert info.n_items > info.n_groups
+    assert rel_err(o, ref) < TOL
+
+
 def test_multi_layer_strides():
     rbs = [(64, 2), (32, 3), (48, 2), (128, 1)] * 2
     srcs = [synth.HeadSource(46, l, h, side, (0.3, 2.5)) for side in (0, 1) for l in range(2) for h in range(2)]
