@@ -34,7 +34,7 @@ sys.path.insert(0, ROOT)
 METRIC = "decode-attn effective HBM GB/s over packed cache (% of peak); compress tok/s"
 FALLBACK_HBM_GBS = 6800.0
 PROFILE = os.path.join(ROOT, "profiles", "decode_scan_llama3_8b.txt")
-CONFIG3_PROFILE = os.path.join(ROOT, "profiles", "decode_scan_llama3_70b_joint.txt")
+JOINT70B_PROFILE = os.path.join(ROOT, "profiles", "decode_scan_llama3_70b_joint.txt")
 SCAN_SOURCES = ["paper_2609_24298_gb300/csrc/decode.cuh", "paper_2609_24298_gb300/csrc/common.cuh"]
 CFG = 2
 SAMPLE_R, SAMPLE_B = 64, 2  # (r, b) of the oracle sample heads: the most common point at 1 bpd
@@ -61,9 +61,13 @@ def parse_args():
     ap.add_argument("--calibration-only", action="store_true", help="only the device calibration leg")
     ap.add_argument("--no-rope", action="store_true", help="skip the RoPE decode leg")
     ap.add_argument("--rope-steps", type=int, default=20, help="timed calls of the RoPE decode leg")
-    ap.add_argument("--no-configs", action="store_true", help="skip the config 1, 3 and 5 decode legs")
-    ap.add_argument("--configs-only", default=None, help="only these of the config 1, 3, 5 decode legs, e.g. 1,3,5")
-    ap.add_argument("--config-steps", type=int, default=30, help="timed steps of the config 3 and 5 legs")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the tiny, Llama-3-70B-shaped joint and ragged-sweep decode legs")
+    ap.add_argument("--configs-only", default=None,
+                    help="only these of those legs, by their ids in synth.CONFIGS (1 tiny, 3 Llama-3-70B-shaped "
+                         "joint, 5 ragged sweep), e.g. 1,3,5")
+    ap.add_argument("--config-steps", type=int, default=30,
+                    help="timed steps of the Llama-3-70B-shaped and ragged-sweep legs")
     return ap.parse_args()
 
 
@@ -646,7 +650,7 @@ def run_rope_leg(args, dev, stream, hp, wl, desc, ws, info, q, lens, out, cpu_ba
 
 
 # ---------------------------------------------------------------------------------------
-# the other decode workloads (configs 1, 3 and 5), measured after the headline
+# the other decode workloads (tiny, Llama-3-70B-shaped joint, ragged sweep), measured after the headline
 # ---------------------------------------------------------------------------------------
 def allocated_params(cfg: int, layers: int, bpd: float, base=None):
     """Per-head parameters of a config at `bpd`: calibration (reused from `base` when given:
@@ -825,7 +829,7 @@ def workload_leg(args, dev, stream, cfg: int, bpd: float, lens, paged: bool, ste
     return out, (hp, srcs)
 
 
-def run_config3_leg(args, dev, stream, cpu_baseline: bool):
+def run_llama3_70b_joint_leg(args, dev, stream, cpu_baseline: bool):
     """Llama-3-70B-shaped joint K+V at 0.5 bpd: 80 layers x 8 kv heads, GQA 8, one 131072-token
     sequence; the step appends the new token and decodes over all layers."""
     from paper_2609_24298_gb300 import synth
@@ -834,11 +838,11 @@ def run_config3_leg(args, dev, stream, cpu_baseline: bool):
     out, _ = workload_leg(args, dev, stream, 3, spec["bpd"], [spec["tokens"]], False, args.config_steps,
                           cpu_baseline, label="llama3-70b-shaped decode step: 80 layers x 8 kv heads (GQA 8) x 1 "
                                               "sequence x 131072 tokens, K and V allocated jointly at 0.5 bpd")
-    out["roofline"]["traffic"] = profiled_traffic(CONFIG3_PROFILE, SCAN_SOURCES)
+    out["roofline"]["traffic"] = profiled_traffic(JOINT70B_PROFILE, SCAN_SOURCES)
     return out
 
 
-def run_config5_leg(args, dev, stream, cpu_baseline: bool):
+def run_ragged_sweep_leg(args, dev, stream, cpu_baseline: bool):
     """Ragged paged rate sweep: 32 layers x 8 kv heads x 32 sequences of lengths uniform in
     [1024, 65536] in 256-token pages (shuffled), every bpd point re-allocated."""
     from paper_2609_24298_gb300 import synth
@@ -852,10 +856,11 @@ def run_config5_leg(args, dev, stream, cpu_baseline: bool):
                                                 f"(lengths in [1024, 65536], sum {int(lens.sum())}), 256-token "
                                                 f"pages, K and V at {bpd} bpd")
         points.append(o)
-    return {"workload": "ragged paged rate sweep (configs[4] shape)", "points": points}
+    return {"workload": "ragged paged rate sweep: 32 layers x 8 kv heads x 32 sequences of 1024-65536 tokens, "
+                        "256-token pages, 0.5 to 4 bpd", "points": points}
 
 
-def run_config1_leg(args, dev, stream, cpu_baseline: bool):
+def run_tiny_leg(args, dev, stream, cpu_baseline: bool):
     """The tiny single-layer case: 8 kv heads, GQA 4, one 2048-token sequence at 2 bpd; the
     decode step's latency."""
     from paper_2609_24298_gb300 import synth
@@ -942,8 +947,8 @@ def run_cobra(args):
         legs = AuxLegs(torch.cuda.current_stream())
         st, cb = torch.cuda.current_stream(), not args.no_cpu_baseline
         todo = {int(x) for x in args.configs_only.split(",")}
-        fns = {1: ("config1_tiny", run_config1_leg), 3: ("config3_llama3_70b_joint", run_config3_leg),
-               5: ("config5_ragged_sweep", run_config5_leg)}
+        fns = {1: ("tiny_2bpd", run_tiny_leg), 3: ("llama3_70b_joint_0p5bpd", run_llama3_70b_joint_leg),
+               5: ("ragged_paged_sweep", run_ragged_sweep_leg)}
         print(json.dumps({name: legs.run(fn, args, dev, st, cb) for c, (name, fn) in fns.items() if c in todo}),
               flush=True)
         return
@@ -1121,9 +1126,9 @@ def run_cobra(args):
     configs = None
     if not args.no_configs and rank == 0:
         cb = not args.no_cpu_baseline and world == 1
-        configs = {"config1_tiny": legs.run(run_config1_leg, args, dev, stream, cb),
-                   "config3_llama3_70b_joint": legs.run(run_config3_leg, args, dev, stream, cb),
-                   "config5_ragged_sweep": legs.run(run_config5_leg, args, dev, stream, cb)}
+        configs = {"tiny_2bpd": legs.run(run_tiny_leg, args, dev, stream, cb),
+                   "llama3_70b_joint_0p5bpd": legs.run(run_llama3_70b_joint_leg, args, dev, stream, cb),
+                   "ragged_paged_sweep": legs.run(run_ragged_sweep_leg, args, dev, stream, cb)}
     compress = None
     if not args.no_compress:
         del hin, hout
@@ -1141,7 +1146,7 @@ def run_cobra(args):
                          "traffic": traffic, "scan_ms": scan_ms,
                          "algorithmic_bytes_per_launch": bytes_step, "frac_of_nominal_8TBs": achieved / 8000.0},
             "compress": compress,
-            "other_decode_configs": configs,
+            "other_decode_workloads": configs,
             "rope": rope,
             "measured": measured,
             "calibration": calibration,

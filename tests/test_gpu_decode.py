@@ -107,7 +107,7 @@ def mixed_heads(kv, rbs, cfg=31, layers=1):
 
 
 def test_tiny_config_full():
-    """Config 1: 1 layer, 8 KV heads, 32 query heads, 2048 tokens, oracle allocation at 2 bpd."""
+    """The tiny workload: 1 layer, 8 KV heads, 32 query heads, 2048 tokens, oracle allocation at 2 bpd."""
     params, srcs = oracle_heads_allocated(1, 1, 2.0)
     o, ref, _ = run_decode(params, srcs, 1, 8, 4, [2048])
     assert rel_err(o, ref) < TOL
