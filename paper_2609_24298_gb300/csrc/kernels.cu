@@ -336,8 +336,14 @@ cobra_status decode_args(const void* params, const cobra_decode_desc* d, const c
   a.pages_per_seq = d->pages_per_seq;
   a.one = kOneH2;
   const int rowb = info->max_row_bytes > 0 ? info->max_row_bytes : 16;
-  // 8 KB of row staging per warp, or two of the largest rows if those are bigger
-  a.ring_bytes = (int)std::max<size_t>(8192, 2 * align_up((size_t)rowb, 128));
+  // 8 KB of row staging per warp, or two of the largest rows if those are bigger.  Rows of
+  // 12 KB and more get four (at most 48 KB, which keeps a CTA within shared memory): with such
+  // rows the copies, not the warps, bound the scan, and three stages of a typical row pair for
+  // 4 warps per SM beat one stage for 8 (a 4 bpd rate sweep measured 0.50 against 0.43 of the
+  // HBM peak; at 3 bpd, with 10 KB rows, the opposite held).
+  size_t ring = std::max<size_t>(8192, 2 * align_up((size_t)rowb, 128));
+  if (rowb >= 12288) ring = std::max(ring, std::min<size_t>(4 * align_up((size_t)rowb, 128), 48 * 1024));
+  a.ring_bytes = (int)ring;
   const long long n_heads = (long long)d->n_layers * d->n_kv_heads;
   if (n_heads * d->n_seqs != info->n_groups) return COBRA_EINVAL;  // plan made for another descriptor
   return COBRA_OK;
