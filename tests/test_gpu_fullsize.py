@@ -115,8 +115,8 @@ def run_workload(cfg, layers, params, srcs, lens, samples, paged=False, seed=5):
     torch.cuda.synchronize()
     assert cobra.cobra_check(stream) == cobra.COBRA_OK
 
-    # the one-call decode step (V append, query projection fused with the K append, scan,
-    # combine) writes the same cache bytes and the same outputs as the separate calls
+    # the one-call decode step (query projection fused with the K and V appends, scan, combine)
+    # writes the same cache bytes and the same outputs as the separate calls
     step_out = torch.full((L, S, H * G, D), float("nan"), dtype=torch.float32, device=DEV)
     cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], xk, xv, pos, q, before, lens_d, pt, step_out, ws,
                             nws, stream)
@@ -135,7 +135,22 @@ def run_workload(cfg, layers, params, srcs, lens, samples, paged=False, seed=5):
     assert torch.equal(host_cache, cache)
     assert torch.equal(step_out, staged_out)
     assert torch.equal(host_out, staged_out.cpu())
-    del before, step_out, staged_out, host_cache, pre
+    # the step can be captured in a CUDA graph (a serving loop's replay): one replay writes the
+    # same cache bytes and the same outputs as the eager call
+    graph_cache = pre.clone()
+    graph_out = torch.full_like(step_out, float("nan"))
+    g = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream()
+    cap.wait_stream(stream)
+    with torch.cuda.graph(g, stream=cap):
+        cobra.cobra_decode_step(block, desc, info, adesc[0], adesc[1], xk, xv, pos, q, graph_cache, lens_d, pt,
+                                graph_out, ws, nws, torch.cuda.current_stream())
+    g.replay()
+    torch.cuda.synchronize()
+    assert cobra.cobra_check(stream) == cobra.COBRA_OK
+    assert torch.equal(graph_cache, cache)
+    assert torch.equal(graph_out, staged_out)
+    del before, step_out, staged_out, host_cache, pre, graph_cache, graph_out, g
 
     # compress + append parity on the sampled heads, then the oracle's rows in their place
     hk, hv = xk.float().cpu().numpy(), xv.float().cpu().numpy()
