@@ -101,7 +101,6 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, uint32_t (&v)[32]) {
       : "r"(taddr)
       : "memory");
 }
-__device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 // 16 consecutive TMEM columns of the warp's 32 lanes: column (taddr + j) of this lane = v[j]
 __device__ __forceinline__ void tc_st32x16(uint32_t taddr, const uint32_t (&v)[16]) {
   asm volatile(
@@ -112,8 +111,8 @@ __device__ __forceinline__ void tc_st32x16(uint32_t taddr, const uint32_t (&v)[1
       : "memory");
 }
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
-// The same wait, with v (the destination of the load in flight) passed through it, so that no
-// use of v can be scheduled ahead of the wait.
+// Wait for this thread's TMEM loads, with v (the destination of the load in flight) passed
+// through the wait, so that no use of v can be scheduled ahead of it.
 __device__ __forceinline__ void tc_wait_ld(uint32_t (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : "+r"(v[0]), "+r"(v[1]), "+r"(v[2]), "+r"(v[3]), "+r"(v[4]), "+r"(v[5]), "+r"(v[6]), "+r"(v[7]),
